@@ -1,0 +1,147 @@
+"""The five Skip-Conv workloads: layer shapes, stacks and seeded inputs.
+
+c0  single 3x3 layer, 32->32 channels, 64x64, T=8, fp32, 1x1 gate blocks, eps 0.05
+c1  single 3x3 layer, 64->64, 128x128, T=16, bf16, 8x8 blocks, eps 0.05
+c2  HRNet-W32-like pose stack on 256x192, T=32, bf16, 4x4 blocks, eps 0.05
+c3  EfficientDet-D0-like MBConv stack at 64x64x40 (1/8 of 512x512), T=32, bf16,
+    8x8 blocks, eps 0.03
+c4  single 3x3 layer, 256->256, 8 streams of 128x128, T=32, bf16, 8x8 blocks,
+    eps 0.05, with a per-frame changed-block density d
+
+Seeds are 1000*config + stream.  Every dimension can be scaled down through
+``make_workload(..., scale=...)`` style overrides for the small parity cases.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+from .video import (block_perturbation_video, he_weights, moving_rect_video,
+                    moving_squares_video, round_to_bf16, traffic_video)
+
+ACT_NONE, ACT_RELU, ACT_SILU = 0, 1, 2
+
+
+@dataclass
+class LayerDef:
+    """One Skip-Conv layer of a workload.  `shortcut` names the index of the
+    stack tensor added before the activation (-1: none; 0 is the stack input,
+    l+1 the output of layer l)."""
+    c_in: int
+    c_out: int
+    k: int
+    stride: int
+    pad: int
+    groups: int
+    block: int
+    eps: float
+    act: int = ACT_NONE
+    shortcut: int = -1
+    name: str = ""
+
+
+@dataclass
+class Workload:
+    name: str
+    dtype: str                      # "f32" or "bf16" (frames, weights, layer outputs)
+    n: int                          # independent streams
+    h: int
+    w: int
+    c: int
+    T: int
+    layers: list
+    weights: list = field(default_factory=list)   # float32 arrays, [c_out][c_in/g][k][k]
+    biases: list = field(default_factory=list)    # float32 arrays or None
+    frames: object = None           # float32 [T, n, h, w, c] or an iterable of (t, frame)
+
+
+def _weights(seed: int, layers, bf16: bool, bias_std: float):
+    rng = np.random.default_rng(seed)
+    ws, bs = [], []
+    for L in layers:
+        ws.append(he_weights(rng, L.c_out, L.c_in // L.groups, L.k, bf16))
+        if bias_std > 0:
+            b = (rng.standard_normal(L.c_out) * bias_std).astype(np.float32)
+            bs.append(round_to_bf16(b) if bf16 else b)
+        else:
+            bs.append(None)
+    return ws, bs
+
+
+def c0(T: int = 8, h: int = 64, w: int = 64, c: int = 32) -> Workload:
+    layers = [LayerDef(c, c, 3, 1, 1, 1, 1, 0.05, name="conv3x3")]
+    frames = moving_squares_video(0, T, h, w, c, n_squares=3, size=8, speed=2, noise_std=0.01)
+    ws, bs = _weights(1, layers, bf16=False, bias_std=0.0)
+    return Workload("c0", "f32", 1, h, w, c, T, layers, ws, bs, frames[:, None])
+
+
+def c1(T: int = 16, h: int = 128, w: int = 128, c: int = 64, n_squares: int = 6, size: int = 16) -> Workload:
+    layers = [LayerDef(c, c, 3, 1, 1, 1, 8, 0.05, name="conv3x3")]
+    frames = round_to_bf16(moving_squares_video(1000, T, h, w, c, n_squares=n_squares, size=size,
+                                                speed=2, noise_std=0.01))
+    ws, bs = _weights(1001, layers, bf16=True, bias_std=0.0)
+    return Workload("c1", "bf16", 1, h, w, c, T, layers, ws, bs, frames[:, None])
+
+
+def c2_layers(block: int = 4, eps: float = 0.05, width: int = 32, stem: int = 64, n_blocks: int = 4):
+    L = [LayerDef(3, stem, 3, 2, 1, 1, block, eps, ACT_RELU, name="stem1"),
+         LayerDef(stem, stem, 3, 2, 1, 1, block, eps, ACT_RELU, name="stem2"),
+         LayerDef(stem, width, 3, 1, 1, 1, block, eps, ACT_RELU, name="transition")]
+    for bi in range(n_blocks):
+        inp = len(L)                        # stack index of this basic block's input
+        L.append(LayerDef(width, width, 3, 1, 1, 1, block, eps, ACT_RELU, name=f"block{bi}.conv1"))
+        L.append(LayerDef(width, width, 3, 1, 1, 1, block, eps, ACT_RELU, shortcut=inp,
+                          name=f"block{bi}.conv2"))
+    return L
+
+
+def c2(T: int = 32, h: int = 256, w: int = 192, n_blocks: int = 4) -> Workload:
+    layers = c2_layers(n_blocks=n_blocks)
+    frames = round_to_bf16(moving_rect_video(2000, T, h, w, 3, n_rects=2, rh=48, rw=32, speed=2, jitter=1))
+    ws, bs = _weights(2001, layers, bf16=True, bias_std=0.01)
+    return Workload("c2", "bf16", 1, h, w, 3, T, layers, ws, bs, frames[:, None])
+
+
+def c3_layers(block: int = 8, eps: float = 0.03, c: int = 40, expand: int = 240, n_blocks: int = 3):
+    L = []
+    for bi in range(n_blocks):
+        inp = len(L)
+        L.append(LayerDef(c, expand, 1, 1, 0, 1, block, eps, ACT_SILU, name=f"mb{bi}.expand"))
+        L.append(LayerDef(expand, expand, 3, 1, 1, expand, block, eps, ACT_SILU, name=f"mb{bi}.dw"))
+        L.append(LayerDef(expand, c, 1, 1, 0, 1, block, eps, ACT_NONE, shortcut=inp, name=f"mb{bi}.project"))
+    return L
+
+
+def c3(T: int = 32, n_blocks: int = 3) -> Workload:
+    """512x512x3 traffic-like video, 8x8 average-pooled to 64x64x3 and lifted
+    to 40 channels by a fixed seeded 1x1 map (input preparation, untimed)."""
+    raw = traffic_video(3000, T)
+    pooled = raw.reshape(T, 64, 8, 64, 8, 3).mean(axis=(2, 4), dtype=np.float64).astype(np.float32)
+    rng = np.random.default_rng(3002)
+    lift = (rng.standard_normal((3, 40)) / np.sqrt(3.0)).astype(np.float32)
+    frames = round_to_bf16(np.einsum("thwc,cd->thwd", pooled, lift).astype(np.float32))
+    layers = c3_layers(n_blocks=n_blocks)
+    ws, bs = _weights(3001, layers, bf16=True, bias_std=0.01)
+    return Workload("c3", "bf16", 1, 64, 64, 40, T, layers, ws, bs, frames[:, None])
+
+
+C4_DENSITIES = (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00)
+
+
+def c4(density: float = 0.10, T: int = 32, n: int = 8, h: int = 128, w: int = 128, c: int = 256,
+       block: int = 8, dtype: str = "bf16") -> Workload:
+    """Density sweep layer.  `frames` is an iterable yielding (t, frame)."""
+    layers = [LayerDef(c, c, 3, 1, 1, 1, block, 0.05, name="conv3x3")]
+    n_changed = int(round(density * (h // block) * (w // block)))
+    bf16 = dtype == "bf16"
+    frames = block_perturbation_video(4000, T, n, h, w, c, block, n_changed, bf16=bf16)
+    ws, bs = _weights(4001, layers, bf16=bf16, bias_std=0.0)
+    return Workload("c4", dtype, n, h, w, c, T, layers, ws, bs, frames)
+
+
+WORKLOADS = {"c0": c0, "c1": c1, "c2": c2, "c3": c3, "c4": c4}
+
+
+def make_workload(name: str, **kw) -> Workload:
+    return WORKLOADS[name](**kw)
