@@ -1,0 +1,414 @@
+#!/usr/bin/env python
+"""Skip-Conv layer-step benchmark on GB300.
+
+Workload (one "step" = one Skip-Conv layer step over one batch):
+  3x3 Skip-Conv layer, 256 -> 256 channels, 8 independent streams of 128x128
+  frames, bf16 storage with fp32 accumulation, 8x8 gate blocks, eps 0.05,
+  Input-Norm gate (mean over the support), with exactly 10% of the blocks of
+  every stream changing per frame (synthetic video, seeded).
+
+Reports stream-frames/s (value), effective TFLOP/s on the active locations,
+the step's roofline fraction, the dominant kernel's roofline, an end-to-end
+number through the host-buffer ABI call, the CPU oracle on the host cores,
+and a density sweep against the library's all-ones dense mode.
+
+    python bench.py [--steps K] [--warmup W] [--impl ours|reference] [--no-sweep]
+Under torchrun every rank runs an independent replica (weak scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Skip-Conv frames/s and effective TFLOP/s vs roofline at measured gate density"
+UNIT = "stream-frames/s"
+N_STREAMS, H, W, C, K, BLOCK, EPS = 8, 128, 128, 256, 3, 8, 0.05
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNELS = ("gate_pixel", "gate_block", "conv", "y_refresh")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--density", type=float, default=0.10)
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--sweep-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+def workload_config(density):
+    return {"workload": "c4: 3x3 Skip-Conv 256->256, %d streams x %dx%d, bf16 (fp32 accum), %dx%d blocks, "
+                        "eps %.2g, %g%% block density" % (N_STREAMS, H, W, BLOCK, BLOCK, EPS, density * 100),
+            "streams": N_STREAMS, "h": H, "w": W, "c_in": C, "c_out": C, "k": K, "block": BLOCK, "eps": EPS,
+            "gate": "input-norm (mean over support)", "density": density,
+            "l2": "flushed between timed steps (256 MiB write)", "parallelism": "replicas"}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+class Clocks:
+    """nvidia-smi sampling during the timed regions."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.proc, self.path = index, None, None
+
+    def start(self):
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_%d.csv" % os.getpid())
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons, power = [], [], set(), []
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None, "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------- workloads
+def device_frames(density, n_frames, rank, torch):
+    import synth
+    wl = synth.make_workload("c4", density=density, T=n_frames, n=N_STREAMS, h=H, w=W, c=C, block=BLOCK,
+                             stream_offset=rank * N_STREAMS)
+    frames, changed = [], []
+    prev = None
+    for t, f in wl.frames:
+        x = torch.from_numpy(f).cuda().to(torch.bfloat16)        # bf16-exact values: no rounding
+        if prev is not None:
+            changed.append(int((x != prev).any(dim=-1).sum().item()))
+        frames.append(x)
+        prev = x
+    return wl, frames, changed
+
+
+def algorithmic(density_active_blocks, changed_pixels, macs_per_block):
+    """Per-step algorithmic bytes and FLOPs of the layer step (c4 shapes)."""
+    x_bytes = N_STREAMS * H * W * C * 2
+    z_block_bytes = BLOCK * BLOCK * C * 4
+    w_bytes = C * C * K * K * 2
+    b_alg = 2 * x_bytes + changed_pixels * C * 2 + 2 * density_active_blocks * z_block_bytes + w_bytes
+    flops = 2.0 * macs_per_block * density_active_blocks
+    gate_bytes = 2 * x_bytes + changed_pixels * C * 2
+    return b_alg, flops, gate_bytes
+
+
+def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
+    """Key frame + `warmup` untimed steps, then `steps` timed steps with an L2
+    flush between them (outside the events).  Returns per-step ms, per-kernel
+    (launches, ms) when profile=True, and the active-block counts."""
+    from paper_2104_11487_gb300 import skipconv_profile, skipconv_profile_read
+    stream = layer.stream
+    layer.reset()
+    t0 = time.perf_counter()
+    layer.step(frames[0])
+    torch.cuda.synchronize()
+    key_ms = (time.perf_counter() - t0) * 1e3
+    for i in range(1, warmup + 1):
+        layer.step(frames[i])
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    counts = []
+    skipconv_profile(layer.handle, profile)
+    for i in range(steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        layer.step(frames[warmup + 1 + i])
+        ev[i][1].record(stream)
+        if profile:
+            counts.append(layer.gate()[2])
+    torch.cuda.synchronize()
+    launches, kms = skipconv_profile_read(layer.handle)
+    ms = [a.elapsed_time(b) for a, b in ev]
+    return ms, launches, kms, counts, key_ms
+
+
+def make_layer(wl, torch, dense_mode=False):
+    from paper_2104_11487_gb300 import SkipConvLayer
+    return SkipConvLayer(N_STREAMS, C, C, H, W, k=K, stride=1, pad=1, block=BLOCK, eps=EPS, dtype="bf16",
+                         dense_mode=dense_mode, weights=torch.from_numpy(wl.weights[0]), bias=None)
+
+
+def traffic_from_profiles(kernel):
+    """dram bytes per launch from the committed ncu summary of `kernel` on
+    this workload, when one exists for the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "%s_c4_d10.md" % kernel)
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        if line.startswith("dram_bytes_per_launch:"):
+            try:
+                return float(line.split(":", 1)[1].split()[0])
+            except ValueError:
+                return None
+    return None
+
+
+# ----------------------------------------------------------- CPU oracle
+def cpu_oracle_sample(seconds, density, max_frames=40):
+    """The oracle as it stands, on the host cores: stream 0 of the same
+    workload, state preset to the frame before the sample (no key frame),
+    stepping frames until `seconds` of work or `max_frames`."""
+    import oracle
+    import synth
+    wl = synth.make_workload("c4", density=density, T=max_frames + 2, n=1, h=H, w=W, c=C, block=BLOCK)
+    spec = oracle.LayerSpec(n=1, c_in=C, c_out=C, h=H, w=W, k=K, block=BLOCK, eps=EPS)
+    lay = oracle.OracleLayer(spec, wl.weights[0], None)
+    it = iter(wl.frames)
+    _, f0 = next(it)
+    lay.x_prev[...] = f0
+    lay.key = False
+    done, t_total = 0, 0.0
+    for _, f in it:
+        x = np.asarray(f, np.float64)
+        t0 = time.perf_counter()
+        lay.step(x)
+        t_total += time.perf_counter() - t0
+        done += 1
+        if t_total >= seconds:
+            break
+    return {"value": done / t_total, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": "stream 0 of the workload, %d frames after a preset state (no key frame), %.1f s, "
+                      "double-precision C loops" % (done, t_total)}
+
+
+# ---------------------------------------------------------------- main
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        return run_reference(args)
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(v):
+        if not dist:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    from paper_2104_11487_gb300 import _lib, skipconv_get_info
+    _lib.lib()
+    pk, pk_src = peaks()
+    hbm, tc_peak = pk["hbm_gbs"], pk["bf16_tflops"]
+
+    n_frames = args.warmup + args.steps + 1
+    wl, frames, changed = device_frames(args.density, n_frames, rank, torch)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    layer = make_layer(wl, torch)
+    info = skipconv_get_info(layer.handle)
+
+    # 1) headline: timed steps, no per-kernel events
+    clocks = Clocks(local)
+    barrier()
+    clocks.start()
+    ms, launches, _, _, key_ms = run_layer_timed(layer, frames, args.warmup, args.steps, flush, torch)
+    barrier()
+    clk = clocks.stop()
+    total_ms = max_over_ranks(sum(ms))
+    ms_per_step = total_ms / args.steps
+    value = world * N_STREAMS * args.steps / (total_ms / 1e3)
+
+    # 2) the same steps with per-kernel CUDA events (dominant kernel's roofline)
+    ms_p, launches_p, kms, counts, _ = run_layer_timed(layer, frames, args.warmup, args.steps, flush, torch,
+                                                       profile=True)
+    active = statistics.mean(counts) if counts else 0.0
+    chg = statistics.mean(changed[args.warmup:args.warmup + args.steps]) if changed else 0.0
+    macs_per_block = BLOCK * BLOCK * C * C * K * K
+    b_alg, flops, gate_bytes = algorithmic(active, chg, macs_per_block)
+    t_step = ms_per_step / 1e3
+    t_roof = max(flops / (tc_peak * 1e12), b_alg / (hbm * 1e9))
+    per_kernel = {KERNELS[k]: {"launches": launches_p[k], "avg_us": (kms[k] / launches_p[k] * 1e3)
+                               if launches_p[k] else None} for k in range(4)}
+    dom = max(range(3), key=lambda k: kms[k])
+    dom_us = kms[dom] / max(1, launches_p[dom]) * 1e3
+    if dom == 2:
+        ach = flops / (dom_us * 1e-6) / 1e12
+        roof = {"kernel": "conv", "bound": "tensor", "achieved": ach, "peak": tc_peak, "unit": "TFLOP/s",
+                "frac": ach / tc_peak, "peak_source": pk_src + " bf16_tflops (burst)",
+                "traffic": traffic_from_profiles("conv")}
+    else:
+        ach = gate_bytes / (dom_us * 1e-6) / 1e9 if dom == 0 else None
+        roof = {"kernel": KERNELS[dom], "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                "frac": (ach / hbm) if ach else None, "peak_source": pk_src + " hbm_gbs",
+                "algorithmic_bytes_per_launch": gate_bytes, "traffic": traffic_from_profiles(KERNELS[dom])}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded block-perturbation video)",
+            "config": workload_config(args.density),
+            "conv_path": {1: "cuda-core", 2: "tensor-core"}.get(info.conv_path),
+            "active_blocks_per_step": active, "block_density_measured": active / (N_STREAMS * (H // BLOCK) ** 2),
+            "changed_pixels_per_step": chg,
+            "eff_tflops": flops / t_step / 1e12,
+            "step_roofline": {"t_roof_us": t_roof * 1e6, "t_meas_us": t_step * 1e6, "frac": t_roof / t_step,
+                              "bytes_alg": b_alg, "flops_active": flops, "peaks": pk_src},
+            "key_frame_ms_host": key_ms,
+            "per_kernel": per_kernel, "roofline": roof,
+            "gpu_launches": int(sum(launches)), "clocks": clk}
+
+    # 3) end to end through the host-buffer ABI call (pinned host frames, z read back)
+    if not args.no_e2e:
+        from paper_2104_11487_gb300 import skipconv_step_host
+        host = [f.cpu().pin_memory() for f in frames]
+        zh = torch.empty((N_STREAMS, H, W, C), dtype=torch.float32).pin_memory()
+        layer.reset()
+        for i in range(args.warmup + 1):
+            skipconv_step_host(layer.handle, host[i], zh)
+        barrier()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            skipconv_step_host(layer.handle, host[args.warmup + 1 + i], zh)
+        t_e2e = max_over_ranks(time.perf_counter() - t0)
+        line["e2e"] = {"value": world * N_STREAMS * args.steps / t_e2e, "unit": UNIT,
+                       "h2d_bytes_per_step": host[0].numel() * 2, "d2h_bytes_per_step": zh.numel() * 4,
+                       "call": "skipconv_step_host (synchronous; host frame in, full fp32 z out)"}
+        del host
+
+    # 4) density sweep vs the all-ones dense mode of the same kernels
+    if not args.no_sweep:
+        sweep = []
+        del frames
+        dense_ms = None
+        for d in (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00):
+            wl_d, fr_d, ch_d = device_frames(d, args.warmup + args.sweep_steps + 1, rank, torch)
+            lay_d = make_layer(wl_d, torch)
+            ms_d, _, _, cnt_d, _ = run_layer_timed(lay_d, fr_d, args.warmup, args.sweep_steps, flush, torch,
+                                                   profile=True)
+            if d == 0.10:
+                lay_dense = make_layer(wl_d, torch, dense_mode=True)
+                ms_dn, _, _, _, _ = run_layer_timed(lay_dense, fr_d, args.warmup, args.sweep_steps, flush, torch)
+                dense_ms = statistics.median(ms_dn)
+                lay_dense.close()
+            act = statistics.mean(cnt_d)
+            chg_d = statistics.mean(ch_d[args.warmup:]) if ch_d else 0.0
+            b_d, f_d, _ = algorithmic(act, chg_d, macs_per_block)
+            t_d = statistics.median(ms_d) / 1e3
+            sweep.append({"density": d, "active_blocks": act, "ms_per_step": t_d * 1e3,
+                          "frames_per_s": N_STREAMS / t_d, "eff_tflops": f_d / t_d / 1e12,
+                          "step_roofline_frac": max(f_d / (tc_peak * 1e12), b_d / (hbm * 1e9)) / t_d})
+            lay_d.close()
+            del fr_d
+        for s in sweep:
+            s["faster_than_dense_mode"] = (s["ms_per_step"] < dense_ms) if dense_ms else None
+        line["sweep"] = {"points": sweep, "dense_mode_ms_per_step": dense_ms}
+
+    # 5) the CPU oracle on the host cores (rank 0, N = 1 only)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_oracle_sample(args.cpu_seconds, args.density)
+    layer.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_reference(args):
+    """The oracle arm: each step is the oracle on a bounded sample of the
+    workload (stream 0, one frame), on the host cores."""
+    import oracle
+    import synth
+    n_frames = args.warmup + args.steps + 1
+    wl = synth.make_workload("c4", density=args.density, T=n_frames + 1, n=1, h=H, w=W, c=C, block=BLOCK)
+    spec = oracle.LayerSpec(n=1, c_in=C, c_out=C, h=H, w=W, k=K, block=BLOCK, eps=EPS)
+    lay = oracle.OracleLayer(spec, wl.weights[0], None)
+    it = iter(wl.frames)
+    _, f0 = next(it)
+    lay.x_prev[...] = f0
+    lay.key = False
+    times = []
+    for i, (_, f) in enumerate(it):
+        x = np.asarray(f, np.float64)
+        t0 = time.perf_counter()
+        lay.step(x)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+        if len(times) >= args.steps:
+            break
+    total = sum(times)
+    value = len(times) / total
+    sample = "oracle (double-precision C loops) on stream 0 of the workload, one frame per step, state preset"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1,
+            "steps": len(times), "warmup": args.warmup, "ms_per_step": total / len(times) * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded block-perturbation video)", "config": workload_config(args.density),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

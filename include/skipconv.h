@@ -1,0 +1,187 @@
+/*
+ * skipconv.h — C ABI of the GB300 (sm_103a) Skip-Convolution layer step.
+ *
+ * Method: Habibian et al., "Skip-Convolutions for Efficient Video Processing",
+ * CVPR 2021 (arXiv 2104.11487).  One handle is one Skip-Conv layer applied to
+ * n_streams independent video streams.  It keeps, per stream, the previous
+ * input x_{t-1} and the output state z~_{t-1}, and each step computes
+ *
+ *     r_t   = x_t - x_{t-1}                                   (Eq. 2)
+ *     g     = block gate of the local l1 norm of r_t           (Eq. 5 / Eq. 7,
+ *             b x b blocks by max-pooling, Sec. 3.2 "Structured Sparsity")
+ *     z~_t  = z~_{t-1} + g (.) (w * r_t)                       (Eq. 3)
+ *
+ * convolving only inside open blocks; closed blocks keep z~_{t-1} untouched.
+ * The first step after create/reset is a key frame (Sec. 3.1: r_1 = x_1,
+ * computed over the whole frame).
+ *
+ * Layouts (all row-major, no padding between rows):
+ *   frames x_t, x_{t-1}, shortcut, y : [n_streams][h][w][c]        (NHWC)
+ *   z                                 : [n_streams][ho][wo][c_out] float32
+ *   weights                           : [c_out][c_in/groups][k_h][k_w] (OIHW)
+ *   block mask                        : [n_streams][nby][nbx] uint8
+ *   active list                       : int32 block ids (n*nby + by)*nbx + bx
+ * with ho = (h + 2*pad - k_h)/stride + 1, wo likewise, nby = ceil(ho/block),
+ * nbx = ceil(wo/block).  Element type of x, shortcut, weights and y is
+ * `dtype` (float32 or bfloat16); z is always float32; bias is float32.
+ *
+ * Execution: every call enqueues work on the CUDA stream given at create and
+ * returns without waiting, except where a function says it synchronises.
+ * Pointers marked "device" must be device-accessible and stay valid until the
+ * enqueued work has completed (stream order).  All functions return a
+ * skipconv_status; no function throws.  A kernel that detects an internal
+ * failure (for example a wait that ran out) records a device error word; the
+ * next ABI call on that handle returns SKIPCONV_ERR_DEVICE.
+ *
+ * Threading: a handle must not be used from two host threads at once.
+ * Different handles are independent.
+ */
+#ifndef SKIPCONV_H
+#define SKIPCONV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SKIPCONV_API __attribute__((visibility("default")))
+#else
+#define SKIPCONV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct skipconv_s* skipconv_handle;
+
+typedef enum {
+    SKIPCONV_OK = 0,
+    SKIPCONV_ERR_INVALID = -1,     /* bad argument, shape or handle            */
+    SKIPCONV_ERR_UNSUPPORTED = -2, /* valid request this build does not cover  */
+    SKIPCONV_ERR_CUDA = -3,        /* a CUDA runtime or driver call failed     */
+    SKIPCONV_ERR_OOM = -4,         /* device or pinned-host allocation failed  */
+    SKIPCONV_ERR_TIMEOUT = -5,     /* a bounded device wait ran out            */
+    SKIPCONV_ERR_DEVICE = -6       /* a kernel recorded an internal error      */
+} skipconv_status;
+
+typedef enum {
+    SKIPCONV_GATE_INPUT_MEAN = 0,  /* Eq. 5, l1 norm / (c_in*k_h*k_w) > eps    */
+    SKIPCONV_GATE_INPUT_SUM = 1,   /* Eq. 5, l1 norm > eps                     */
+    SKIPCONV_GATE_OUTPUT = 2       /* Eq. 7, ||w||_1 * l1 norm > eps            */
+} skipconv_gate;
+
+typedef enum { SKIPCONV_F32 = 0, SKIPCONV_BF16 = 1 } skipconv_dtype;
+
+typedef enum { SKIPCONV_ACT_NONE = 0, SKIPCONV_ACT_RELU = 1, SKIPCONV_ACT_SILU = 2 } skipconv_act;
+
+typedef enum {
+    SKIPCONV_PATH_AUTO = 0,        /* tensor cores where supported, else CUDA cores */
+    SKIPCONV_PATH_CUDA_CORE = 1,   /* float32 FMA direct convolution              */
+    SKIPCONV_PATH_TENSOR_CORE = 2  /* tcgen05 implicit GEMM (bf16 in, fp32 accum)  */
+} skipconv_path;
+
+typedef struct {
+    int n_streams;     /* independent streams advanced together, >= 1              */
+    int c_in, c_out;   /* channels; both divisible by groups                       */
+    int h, w;          /* input frame size                                          */
+    int k_h, k_w;      /* kernel size                                               */
+    int stride;        /* >= 1, both directions                                     */
+    int pad;           /* zero padding, both directions, >= 0                       */
+    int groups;        /* 1 = dense, c_in = c_out = groups: depthwise               */
+    int block;         /* b: gate block edge on the output grid, >= 1               */
+    float eps;         /* gate threshold, >= 0                                      */
+    int gate;          /* skipconv_gate                                             */
+    int dtype;         /* skipconv_dtype of x, shortcut, weights and y              */
+    int activation;    /* skipconv_act applied to y only (z is pre-activation)      */
+    int emit_y;        /* 1: keep y = act(z [+ shortcut]) in dtype for the next layer */
+    int dense_mode;    /* 1: every gate open (in-library dense reference)           */
+    int conv_path;     /* skipconv_path                                             */
+} skipconv_params;
+
+/* Create a layer.  Copies and repacks the weights (device pointer, OIHW,
+ * dtype), copies the optional bias (device float32 [c_out], NULL = 0),
+ * allocates all state on the current device and resets it (next step is a key
+ * frame).  `stream` is a cudaStream_t (NULL = legacy default stream).
+ * Synchronises the stream once.  On failure *out is NULL.
+ * Errors: INVALID (NULL pointer, non-positive or inconsistent sizes, unknown
+ * enum), UNSUPPORTED (conv_path forced to a path that cannot run this shape),
+ * OOM, CUDA. */
+SKIPCONV_API int skipconv_create(const skipconv_params* params, const void* weights_oihw,
+                    const float* bias, void* stream, skipconv_handle* out);
+
+/* Reset the recurrence (Sec. 3.1 key frame; Table 4's reference-frame reset):
+ * x_{t-1} = 0, z = bias, and the next step processes the whole frame.
+ * Enqueued on the handle's stream. */
+SKIPCONV_API int skipconv_reset_state(skipconv_handle h);
+
+/* One Skip-Conv step (Eq. 2, 5/7, 3).  x_t: device frame [n][h][w][c_in] in
+ * dtype, 16-byte aligned.  shortcut: NULL, or a device tensor
+ * [n][ho][wo][c_out] in dtype added to z before the activation when y is
+ * kept (then y is refreshed over the whole frame).  Updates z in place at the
+ * open blocks, the gate outputs, y (if kept) and x_{t-1} <- x_t.  Enqueued;
+ * x_t and shortcut must stay valid until the stream reaches this work. */
+SKIPCONV_API int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut);
+
+/* The same step on host buffers: copies x_t (host, [n][h][w][c_in] dtype;
+ * pinned memory makes the copy asynchronous DMA) to the device, runs the
+ * step, copies the whole z back to z_out (host float32 [n][ho][wo][c_out],
+ * may be NULL to skip the read-back), and synchronises the stream before
+ * returning.  The first call allocates a device staging frame. */
+SKIPCONV_API int skipconv_step_host(skipconv_handle h, const void* x_t_host, float* z_out_host);
+
+/* Synchronise the stream and free everything.  NULL is accepted. */
+SKIPCONV_API int skipconv_destroy(skipconv_handle h);
+
+/* Read-only views of the handle's device state, valid until the next step,
+ * reset or destroy (read them in stream order). */
+SKIPCONV_API int skipconv_get_z(skipconv_handle h, const float** z);
+SKIPCONV_API int skipconv_get_y(skipconv_handle h, const void** y);            /* NULL unless emit_y */
+SKIPCONV_API int skipconv_get_prev_input(skipconv_handle h, const void** x_prev); /* x_{t-1} for the next step */
+/* Gate of the last step: block mask, the compacted list of open block ids
+ * (order unspecified) and its length (device int32). */
+SKIPCONV_API int skipconv_get_gate(skipconv_handle h, const uint8_t** block_mask, const int32_t** active_list,
+                      const int32_t** active_count);
+
+/* Shape facts of a handle (host values). */
+typedef struct {
+    int ho, wo;        /* output frame size                                   */
+    int nby, nbx;      /* gate blocks per stream                              */
+    int conv_path;     /* path actually used: SKIPCONV_PATH_CUDA_CORE or _TENSOR_CORE */
+    int num_sms;       /* SMs of the device the handle lives on               */
+    size_t state_bytes;/* device bytes held by the handle                     */
+} skipconv_info;
+SKIPCONV_API int skipconv_get_info(skipconv_handle h, skipconv_info* info);
+
+/* Statistics of the last step.  Synchronises the stream.  active_blocks is
+ * the number of open blocks over all streams, active_locations the output
+ * locations inside them, macs = active_locations * c_out * (c_in/groups) *
+ * k_h * k_w (the MAC count of Eq. 9's accounting).  Any pointer may be NULL. */
+SKIPCONV_API int skipconv_get_stats(skipconv_handle h, long long* active_blocks, long long* active_locations,
+                       double* macs);
+
+/* Synchronise the stream and report the device error word:
+ * SKIPCONV_OK, SKIPCONV_ERR_TIMEOUT or SKIPCONV_ERR_DEVICE. */
+SKIPCONV_API int skipconv_check_device(skipconv_handle h);
+
+/* Per-kernel timing.  Kernel kinds: 0 gate_pixel (residual, channel l1 norm,
+ * state commit), 1 gate_block (support norm, block gate, compaction), 2 the
+ * convolution of the open blocks (either path), 3 y refresh.  Launch counts
+ * are always kept; with enable = 1 each launch is also bracketed by CUDA
+ * events on the handle's stream.  skipconv_profile resets both. */
+SKIPCONV_API int skipconv_profile(skipconv_handle h, int enable);
+/* Synchronise the stream and report, per kernel kind (arrays of 4), the
+ * launches and the summed event-timed milliseconds since skipconv_profile
+ * (milliseconds are 0 unless timing was enabled). */
+SKIPCONV_API int skipconv_profile_read(skipconv_handle h, long long* launches, double* ms);
+
+/* Human-readable name of a status code (static string). */
+SKIPCONV_API const char* skipconv_status_string(int status);
+
+/* Detail of the last failure on the calling thread (static per thread). */
+SKIPCONV_API const char* skipconv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SKIPCONV_H */

@@ -1,0 +1,553 @@
+// Host side of the Skip-Conv C ABI (include/skipconv.h): argument checks,
+// state allocation, weight repacking, and the per-step launch sequence
+//   gate_pixel -> gate_block -> conv (tensor-core or CUDA-core) [-> y_refresh]
+// all on the handle's stream, with no host synchronisation per step.
+#include <stdarg.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <new>
+
+#include "sc_internal.h"
+
+namespace sc {
+
+int gate_max_channels(int dtype, bool vec);
+
+static thread_local char g_last_error[512];
+
+void set_error(const char* fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+    va_end(ap);
+}
+
+EncodeTiledFn encode_tiled_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)p;
+    }
+    return fn;
+}
+
+// Host-side fault injection for the cleanup paths: SKIPCONV_FAULT_ALLOC=k
+// makes the k-th device allocation of skipconv_create fail (k >= 1).
+static int fault_alloc_index()
+{
+    const char* s = getenv("SKIPCONV_FAULT_ALLOC");
+    return s ? atoi(s) : 0;
+}
+
+struct Allocator {
+    int counter = 0;
+    int fail_at = 0;
+    size_t bytes = 0;
+    cudaError_t dev(void** p, size_t n)
+    {
+        ++counter;
+        if (fail_at > 0 && counter == fail_at) {
+            *p = nullptr;
+            return cudaErrorMemoryAllocation;
+        }
+        cudaError_t e = cudaMalloc(p, n < 16 ? 16 : n);
+        if (e == cudaSuccess) bytes += n;
+        return e;
+    }
+};
+
+static void prof_release(Layer* L)
+{
+    if (L->prof_ev) {
+        for (int i = 0; i < 2 * L->prof_cap; ++i)
+            if (L->prof_ev[i]) cudaEventDestroy(L->prof_ev[i]);
+        free(L->prof_ev);
+    }
+    free(L->prof_kind);
+    L->prof_ev = nullptr;
+    L->prof_kind = nullptr;
+    L->prof_cap = L->prof_n = 0;
+}
+
+// Record the event opening a timed launch of `kind`; returns the slot or -1.
+static int prof_begin(Layer* L, int kind)
+{
+    L->launches[kind] += 1;
+    if (!L->prof_on) return -1;
+    if (L->prof_n == L->prof_cap) {
+        const int cap = L->prof_cap ? 2 * L->prof_cap : 256;
+        cudaEvent_t* ev = (cudaEvent_t*)calloc(2 * (size_t)cap, sizeof(cudaEvent_t));
+        int* kinds = (int*)calloc(cap, sizeof(int));
+        if (!ev || !kinds) {
+            free(ev);
+            free(kinds);
+            return -1;
+        }
+        if (L->prof_ev) memcpy(ev, L->prof_ev, 2 * (size_t)L->prof_cap * sizeof(cudaEvent_t));
+        if (L->prof_kind) memcpy(kinds, L->prof_kind, (size_t)L->prof_cap * sizeof(int));
+        free(L->prof_ev);
+        free(L->prof_kind);
+        L->prof_ev = ev;
+        L->prof_kind = kinds;
+        L->prof_cap = cap;
+    }
+    const int i = L->prof_n;
+    for (int k = 0; k < 2; ++k)
+        if (!L->prof_ev[2 * i + k] && cudaEventCreate(&L->prof_ev[2 * i + k]) != cudaSuccess) return -1;
+    L->prof_kind[i] = kind;
+    if (cudaEventRecord(L->prof_ev[2 * i], L->stream) != cudaSuccess) return -1;
+    return i;
+}
+
+static void prof_end(Layer* L, int slot)
+{
+    if (slot < 0) return;
+    if (cudaEventRecord(L->prof_ev[2 * slot + 1], L->stream) == cudaSuccess) L->prof_n = slot + 1;
+}
+
+static void free_buffers(Layer* L)
+{
+    prof_release(L);
+    void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
+                    L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    if (L->err_host) cudaFreeHost(L->err_host);
+}
+
+static int status_of(cudaError_t e)
+{
+    if (e == cudaSuccess) return SKIPCONV_OK;
+    cudaGetLastError();  // clear a sticky launch error so the next call starts clean
+    set_error("CUDA error %d: %s", (int)e, cudaGetErrorString(e));
+    return e == cudaErrorMemoryAllocation ? SKIPCONV_ERR_OOM : SKIPCONV_ERR_CUDA;
+}
+
+static int check_device_word(const Layer* L)
+{
+    const int v = *(volatile int*)L->err_host;
+    if (v == DEV_OK) return SKIPCONV_OK;
+    set_error("device error word %d", v);
+    return v == DEV_TIMEOUT ? SKIPCONV_ERR_TIMEOUT : SKIPCONV_ERR_DEVICE;
+}
+
+static int validate(const skipconv_params* p)
+{
+    if (!p) return set_error("params is NULL"), SKIPCONV_ERR_INVALID;
+    if (p->n_streams < 1 || p->c_in < 1 || p->c_out < 1 || p->h < 1 || p->w < 1 || p->k_h < 1 || p->k_w < 1 ||
+        p->stride < 1 || p->pad < 0 || p->groups < 1 || p->block < 1)
+        return set_error("non-positive size in params"), SKIPCONV_ERR_INVALID;
+    if (p->c_in % p->groups || p->c_out % p->groups)
+        return set_error("c_in and c_out must be divisible by groups"), SKIPCONV_ERR_INVALID;
+    if (p->h + 2 * p->pad < p->k_h || p->w + 2 * p->pad < p->k_w)
+        return set_error("kernel larger than the padded frame"), SKIPCONV_ERR_INVALID;
+    if (!(p->eps >= 0.f)) return set_error("eps must be >= 0"), SKIPCONV_ERR_INVALID;
+    if (p->gate < SKIPCONV_GATE_INPUT_MEAN || p->gate > SKIPCONV_GATE_OUTPUT)
+        return set_error("unknown gate %d", p->gate), SKIPCONV_ERR_INVALID;
+    if (p->dtype != SKIPCONV_F32 && p->dtype != SKIPCONV_BF16)
+        return set_error("unknown dtype %d", p->dtype), SKIPCONV_ERR_INVALID;
+    if (p->activation < SKIPCONV_ACT_NONE || p->activation > SKIPCONV_ACT_SILU)
+        return set_error("unknown activation %d", p->activation), SKIPCONV_ERR_INVALID;
+    if (p->conv_path < SKIPCONV_PATH_AUTO || p->conv_path > SKIPCONV_PATH_TENSOR_CORE)
+        return set_error("unknown conv_path %d", p->conv_path), SKIPCONV_ERR_INVALID;
+    const long long frame = (long long)p->n_streams * p->h * p->w;
+    if (frame * p->c_in > (1LL << 40)) return set_error("frame too large"), SKIPCONV_ERR_INVALID;
+    const int ho = (p->h + 2 * p->pad - p->k_h) / p->stride + 1;
+    const int wo = (p->w + 2 * p->pad - p->k_w) / p->stride + 1;
+    const long long nblocks = (long long)p->n_streams * ((ho + p->block - 1) / p->block) * ((wo + p->block - 1) / p->block);
+    if (nblocks >= (1LL << 31)) return set_error("too many gate blocks"), SKIPCONV_ERR_INVALID;
+    if (p->c_in > gate_max_channels(p->dtype, false))
+        return set_error("c_in above %d", gate_max_channels(p->dtype, false)), SKIPCONV_ERR_UNSUPPORTED;
+    return SKIPCONV_OK;
+}
+
+}  // namespace sc
+
+using namespace sc;
+
+struct skipconv_s {
+    Layer L;
+};
+
+static Layer* get(skipconv_handle h) { return h ? &h->L : nullptr; }
+
+extern "C" {
+
+const char* skipconv_status_string(int s)
+{
+    switch (s) {
+    case SKIPCONV_OK: return "SKIPCONV_OK";
+    case SKIPCONV_ERR_INVALID: return "SKIPCONV_ERR_INVALID";
+    case SKIPCONV_ERR_UNSUPPORTED: return "SKIPCONV_ERR_UNSUPPORTED";
+    case SKIPCONV_ERR_CUDA: return "SKIPCONV_ERR_CUDA";
+    case SKIPCONV_ERR_OOM: return "SKIPCONV_ERR_OOM";
+    case SKIPCONV_ERR_TIMEOUT: return "SKIPCONV_ERR_TIMEOUT";
+    case SKIPCONV_ERR_DEVICE: return "SKIPCONV_ERR_DEVICE";
+    default: return "SKIPCONV_UNKNOWN_STATUS";
+    }
+}
+
+const char* skipconv_last_error(void) { return g_last_error; }
+
+int skipconv_create(const skipconv_params* params, const void* weights_oihw, const float* bias, void* stream,
+                    skipconv_handle* out)
+{
+    if (!out) return set_error("out is NULL"), SKIPCONV_ERR_INVALID;
+    *out = nullptr;
+    int st = validate(params);
+    if (st) return st;
+    if (!weights_oihw) return set_error("weights is NULL"), SKIPCONV_ERR_INVALID;
+
+    skipconv_s* h = new (std::nothrow) skipconv_s();
+    if (!h) return set_error("host allocation failed"), SKIPCONV_ERR_OOM;
+    Layer& L = h->L;
+    memset(&L, 0, sizeof(L));
+    L.p = *params;
+    L.stream = (cudaStream_t)stream;
+    L.ho = (L.p.h + 2 * L.p.pad - L.p.k_h) / L.p.stride + 1;
+    L.wo = (L.p.w + 2 * L.p.pad - L.p.k_w) / L.p.stride + 1;
+    L.nby = (L.ho + L.p.block - 1) / L.p.block;
+    L.nbx = (L.wo + L.p.block - 1) / L.p.block;
+    L.cpg = L.p.c_in / L.p.groups;
+    L.opg = L.p.c_out / L.p.groups;
+    L.esize = L.p.dtype == SKIPCONV_BF16 ? 2 : 4;
+
+    cudaError_t e = cudaGetDevice(&L.device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&L.num_sms, cudaDevAttrMultiProcessorCount, L.device);
+    if (e != cudaSuccess) {
+        st = status_of(e);
+        delete h;
+        return st;
+    }
+
+    // choose the convolution path
+    const char* why = "";
+    const bool tc_ok = conv_tc_supported(L.p, &why);
+    if (L.p.conv_path == SKIPCONV_PATH_TENSOR_CORE && !tc_ok) {
+        set_error("tensor-core path unsupported: %s", why);
+        delete h;
+        return SKIPCONV_ERR_UNSUPPORTED;
+    }
+    L.path = (L.p.conv_path == SKIPCONV_PATH_CUDA_CORE || !tc_ok) ? SKIPCONV_PATH_CUDA_CORE
+                                                                   : SKIPCONV_PATH_TENSOR_CORE;
+    if (L.path == SKIPCONV_PATH_CUDA_CORE && conv_cc_smem_bytes(L) > 200 * 1024) {
+        set_error("CUDA-core path: halo tile of %zu bytes exceeds shared memory", conv_cc_smem_bytes(L));
+        delete h;
+        return SKIPCONV_ERR_UNSUPPORTED;
+    }
+    L.ci_pad = ((L.p.c_in + 63) / 64) * 64;
+    L.co_pad = ((L.p.c_out + 127) / 128) * 128;
+
+    Allocator A;
+    A.fail_at = fault_alloc_index();
+    const size_t npix = (size_t)L.p.n_streams * L.p.h * L.p.w;
+    const size_t xbytes = npix * L.p.c_in * L.esize;
+    const size_t nz = (size_t)L.p.n_streams * L.ho * L.wo * L.p.c_out;
+    const size_t nblk = (size_t)L.p.n_streams * L.nby * L.nbx;
+    const size_t nw = (size_t)L.p.c_out * L.cpg * L.p.k_h * L.p.k_w;
+    double* w_l1_dev = nullptr;
+    e = cudaSuccess;
+    if (e == cudaSuccess) e = A.dev(&L.xbuf[0], xbytes);
+    if (e == cudaSuccess) e = A.dev(&L.xbuf[1], xbytes);
+    if (e == cudaSuccess) e = A.dev((void**)&L.chg[0], npix);
+    if (e == cudaSuccess) e = A.dev((void**)&L.chg[1], npix);
+    if (e == cudaSuccess) e = A.dev((void**)&L.pix_l1, npix * sizeof(float));
+    if (e == cudaSuccess) e = A.dev((void**)&L.mask, nblk);
+    if (e == cudaSuccess) e = A.dev((void**)&L.list, nblk * sizeof(int32_t));
+    if (e == cudaSuccess) e = A.dev((void**)&L.counters, 64 * sizeof(int32_t));
+    if (e == cudaSuccess) e = A.dev((void**)&L.z, nz * sizeof(float));
+    if (e == cudaSuccess && L.p.emit_y) e = A.dev(&L.y, nz * L.esize);
+    if (e == cudaSuccess) e = A.dev((void**)&L.bias, L.p.c_out * sizeof(float));
+    if (e == cudaSuccess) e = A.dev((void**)&L.w_cc, nw * sizeof(float));
+    if (e == cudaSuccess && L.path == SKIPCONV_PATH_TENSOR_CORE)
+        e = A.dev((void**)&L.w_tc, (size_t)L.co_pad * L.p.k_h * L.p.k_w * L.ci_pad * sizeof(__nv_bfloat16));
+    if (e == cudaSuccess) e = A.dev((void**)&w_l1_dev, sizeof(double));
+    if (e == cudaSuccess) {
+        e = cudaHostAlloc((void**)&L.err_host, sizeof(int), cudaHostAllocMapped);
+        if (e == cudaSuccess) {
+            *L.err_host = 0;
+            e = cudaHostGetDevicePointer((void**)&L.err_dev, L.err_host, 0);
+        }
+    }
+    L.state_bytes = A.bytes;
+    if (e != cudaSuccess) {
+        st = status_of(e);
+        if (w_l1_dev) cudaFree(w_l1_dev);
+        free_buffers(&h->L);
+        delete h;
+        return st;
+    }
+
+    // weights, bias, ||w||_1
+    double w_l1 = 0.0;
+    e = cudaMemsetAsync(w_l1_dev, 0, sizeof(double), L.stream);
+    if (e == cudaSuccess && L.w_tc)
+        e = cudaMemsetAsync(L.w_tc, 0, (size_t)L.co_pad * L.p.k_h * L.p.k_w * L.ci_pad * sizeof(__nv_bfloat16),
+                            L.stream);
+    if (e == cudaSuccess) e = launch_pack_weights(L, weights_oihw, w_l1_dev);
+    if (e == cudaSuccess) {
+        if (bias)
+            e = cudaMemcpyAsync(L.bias, bias, L.p.c_out * sizeof(float), cudaMemcpyDeviceToDevice, L.stream);
+        else
+            e = cudaMemsetAsync(L.bias, 0, L.p.c_out * sizeof(float), L.stream);
+    }
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&w_l1, w_l1_dev, sizeof(double), cudaMemcpyDeviceToHost, L.stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(L.stream);
+    cudaFree(w_l1_dev);
+    (void)nw;
+
+    // The gate compares the raw local l1 sum S (sum of |r| over the support) with
+    // a threshold equivalent to the chosen normalisation of Eq. 5 / Eq. 7.
+    double thr;
+    if (L.p.gate == SKIPCONV_GATE_INPUT_MEAN) thr = (double)L.p.eps * L.p.c_in * L.p.k_h * L.p.k_w;
+    else if (L.p.gate == SKIPCONV_GATE_INPUT_SUM) thr = (double)L.p.eps;
+    else thr = w_l1 > 0.0 ? (double)L.p.eps / w_l1 : INFINITY;
+    L.gate_thr = (float)thr;
+
+    if (e == cudaSuccess && L.path == SKIPCONV_PATH_TENSOR_CORE) e = conv_tc_prepare(L);
+    if (e == cudaSuccess) {
+        h->L.key = 1;
+        st = skipconv_reset_state(h);
+        if (st == SKIPCONV_OK) e = cudaStreamSynchronize(L.stream);
+        else e = cudaErrorUnknown;
+    }
+    if (e != cudaSuccess) {
+        st = st ? st : status_of(e);
+        free_buffers(&h->L);
+        delete h;
+        return st;
+    }
+    *out = h;
+    return SKIPCONV_OK;
+}
+
+int skipconv_reset_state(skipconv_handle h)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (int st = check_device_word(L)) return st;
+    const size_t npix = (size_t)L->p.n_streams * L->p.h * L->p.w;
+    const size_t xbytes = npix * L->p.c_in * L->esize;
+    cudaError_t e = cudaMemsetAsync(L->xbuf[0], 0, xbytes, L->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->xbuf[1], 0, xbytes, L->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[0], 0, npix, L->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[1], 0, npix, L->stream);
+    if (e == cudaSuccess) e = launch_reset_z(*L);
+    if (e == cudaSuccess && L->y) e = cudaMemsetAsync(L->y, 0, (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * L->esize, L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    L->t = 0;
+    L->key = 1;
+    return SKIPCONV_OK;
+}
+
+int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!x_t) return set_error("x_t is NULL"), SKIPCONV_ERR_INVALID;
+    if ((uintptr_t)x_t % 16 || (uintptr_t)shortcut % 16)
+        return set_error("x_t and shortcut must be 16-byte aligned"), SKIPCONV_ERR_INVALID;
+    if (shortcut && !L->y) return set_error("shortcut given but the layer keeps no y (emit_y = 0)"), SKIPCONV_ERR_INVALID;
+    if (int st = check_device_word(L)) return st;
+    const int cur = (int)(L->t & 1), nxt = cur ^ 1;
+    // xbuf[cur] holds x_{t-1}; xbuf[nxt] holds x_{t-2} and receives x_t.
+    // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
+    int slot = prof_begin(L, 0);
+    cudaError_t e = launch_gate_pixel(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur]);
+    prof_end(L, slot);
+    if (e == cudaSuccess) {
+        slot = prof_begin(L, 1);
+        e = launch_gate_block(*L, (L->key || L->p.dense_mode) ? 1 : 0);
+        prof_end(L, slot);
+    }
+    if (e == cudaSuccess) {
+        slot = prof_begin(L, 2);
+        if (L->path == SKIPCONV_PATH_TENSOR_CORE) e = launch_conv_tc(*L, x_t, L->xbuf[cur], cur);
+        else e = launch_conv_cc(*L, x_t, L->xbuf[cur]);
+        prof_end(L, slot);
+    }
+    if (e == cudaSuccess && L->y && shortcut) {
+        slot = prof_begin(L, 3);
+        e = launch_y_refresh(*L, shortcut);
+        prof_end(L, slot);
+    }
+    if (e != cudaSuccess) return status_of(e);
+    L->t += 1;
+    L->key = 0;
+    return SKIPCONV_OK;
+}
+
+int skipconv_step_host(skipconv_handle h, const void* x_t_host, float* z_out_host)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!x_t_host) return set_error("x_t_host is NULL"), SKIPCONV_ERR_INVALID;
+    const size_t xbytes = (size_t)L->p.n_streams * L->p.h * L->p.w * L->p.c_in * L->esize;
+    cudaError_t e = cudaSuccess;
+    if (!L->x_stage) {
+        e = cudaMalloc(&L->x_stage, xbytes);
+        if (e != cudaSuccess) {
+            L->x_stage = nullptr;
+            return status_of(e);
+        }
+        L->state_bytes += xbytes;
+    }
+    e = cudaMemcpyAsync(L->x_stage, x_t_host, xbytes, cudaMemcpyHostToDevice, L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    int st = skipconv_step(h, L->x_stage, nullptr);
+    if (st) return st;
+    if (z_out_host) {
+        const size_t zbytes = (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * sizeof(float);
+        e = cudaMemcpyAsync(z_out_host, L->z, zbytes, cudaMemcpyDeviceToHost, L->stream);
+        if (e != cudaSuccess) return status_of(e);
+    }
+    e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    return check_device_word(L);
+}
+
+int skipconv_destroy(skipconv_handle h)
+{
+    if (!h) return SKIPCONV_OK;
+    Layer* L = get(h);
+    cudaError_t e = cudaStreamSynchronize(L->stream);
+    int st = e == cudaSuccess ? check_device_word(L) : status_of(e);
+    free_buffers(L);
+    delete h;
+    return st;
+}
+
+int skipconv_get_z(skipconv_handle h, const float** z)
+{
+    Layer* L = get(h);
+    if (!L || !z) return set_error("NULL argument"), SKIPCONV_ERR_INVALID;
+    *z = L->z;
+    return SKIPCONV_OK;
+}
+
+int skipconv_get_y(skipconv_handle h, const void** y)
+{
+    Layer* L = get(h);
+    if (!L || !y) return set_error("NULL argument"), SKIPCONV_ERR_INVALID;
+    *y = L->y;
+    return SKIPCONV_OK;
+}
+
+int skipconv_get_prev_input(skipconv_handle h, const void** x_prev)
+{
+    Layer* L = get(h);
+    if (!L || !x_prev) return set_error("NULL argument"), SKIPCONV_ERR_INVALID;
+    *x_prev = L->xbuf[L->t & 1];
+    return SKIPCONV_OK;
+}
+
+int skipconv_get_gate(skipconv_handle h, const uint8_t** block_mask, const int32_t** active_list,
+                      const int32_t** active_count)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (block_mask) *block_mask = L->mask;
+    if (active_list) *active_list = L->list;
+    if (active_count) *active_count = L->counters;
+    return SKIPCONV_OK;
+}
+
+int skipconv_get_info(skipconv_handle h, skipconv_info* info)
+{
+    Layer* L = get(h);
+    if (!L || !info) return set_error("NULL argument"), SKIPCONV_ERR_INVALID;
+    info->ho = L->ho;
+    info->wo = L->wo;
+    info->nby = L->nby;
+    info->nbx = L->nbx;
+    info->conv_path = L->path;
+    info->num_sms = L->num_sms;
+    info->state_bytes = L->state_bytes;
+    return SKIPCONV_OK;
+}
+
+int skipconv_get_stats(skipconv_handle h, long long* active_blocks, long long* active_locations, double* macs)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    const size_t nblk = (size_t)L->p.n_streams * L->nby * L->nbx;
+    uint8_t* m = (uint8_t*)malloc(nblk);
+    if (!m) return set_error("host allocation failed"), SKIPCONV_ERR_OOM;
+    cudaError_t e = cudaMemcpyAsync(m, L->mask, nblk, cudaMemcpyDeviceToHost, L->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) {
+        free(m);
+        return status_of(e);
+    }
+    long long nb = 0, nloc = 0;
+    for (size_t k = 0; k < nblk; ++k) {
+        if (!m[k]) continue;
+        const int bx = (int)(k % L->nbx), by = (int)((k / L->nbx) % L->nby);
+        const int bh = L->ho - by * L->p.block < L->p.block ? L->ho - by * L->p.block : L->p.block;
+        const int bw = L->wo - bx * L->p.block < L->p.block ? L->wo - bx * L->p.block : L->p.block;
+        ++nb;
+        nloc += (long long)bh * bw;
+    }
+    free(m);
+    if (active_blocks) *active_blocks = nb;
+    if (active_locations) *active_locations = nloc;
+    if (macs) *macs = (double)nloc * L->p.c_out * L->cpg * L->p.k_h * L->p.k_w;
+    return check_device_word(L);
+}
+
+int skipconv_profile(skipconv_handle h, int enable)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    cudaError_t e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    for (int k = 0; k < 4; ++k) {
+        L->launches[k] = 0;
+        L->prof_ms[k] = 0.0;
+    }
+    L->prof_n = 0;
+    L->prof_on = enable ? 1 : 0;
+    return SKIPCONV_OK;
+}
+
+int skipconv_profile_read(skipconv_handle h, long long* launches, double* ms)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    cudaError_t e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    for (int i = 0; i < L->prof_n; ++i) {
+        float t = 0.f;
+        e = cudaEventElapsedTime(&t, L->prof_ev[2 * i], L->prof_ev[2 * i + 1]);
+        if (e != cudaSuccess) return status_of(e);
+        L->prof_ms[L->prof_kind[i]] += t;
+    }
+    L->prof_n = 0;
+    for (int k = 0; k < 4; ++k) {
+        if (launches) launches[k] = L->launches[k];
+        if (ms) ms[k] = L->prof_ms[k];
+    }
+    return SKIPCONV_OK;
+}
+
+int skipconv_check_device(skipconv_handle h)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    cudaError_t e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    return check_device_word(L);
+}
+
+}  // extern "C"

@@ -1,0 +1,111 @@
+// Internal declarations of the Skip-Conv CUDA library (not part of the ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "skipconv.h"
+
+namespace sc {
+
+// Device error word values (written by kernels, read by the host).
+enum : int { DEV_OK = 0, DEV_TIMEOUT = 1, DEV_BAD_INDEX = 2 };
+
+struct Layer {
+    skipconv_params p;
+    int ho, wo, nby, nbx;
+    int cpg, opg;           // input / output channels per group
+    int esize;              // bytes per element of dtype
+    int path;               // SKIPCONV_PATH_CUDA_CORE or SKIPCONV_PATH_TENSOR_CORE
+    int num_sms;
+    int device;
+    cudaStream_t stream;
+    float gate_thr;         // threshold on the raw local l1 sum S (see api)
+
+    // device state
+    void* xbuf[2];          // ping-pong x_{t-1} / x_{t-2} frames, dtype
+    uint8_t* chg[2];        // per input pixel: x_t != x_{t-1}, for the last two steps
+    float* pix_l1;          // per input pixel: sum over channels of |r| (scratch)
+    uint8_t* mask;          // [n][nby][nbx]
+    int32_t* list;          // active block ids
+    int32_t* counters;      // [0] active count, [1..] scratch counters
+    float* z;               // [n][ho][wo][c_out]
+    void* y;                // [n][ho][wo][c_out] dtype or NULL
+    float* bias;            // [c_out]
+    float* w_cc;            // [cpg][k_h][k_w][c_out] fp32 (CUDA-core path)
+    __nv_bfloat16* w_tc;    // [co_pad][k_h*k_w*ci_pad] bf16 (tensor-core path)
+    int ci_pad, co_pad;     // tensor-core padding of c_in (multiple of 64) and c_out (of 128)
+    void* x_stage;          // device staging frame for skipconv_step_host (lazy)
+    size_t state_bytes;
+
+    // error word: pinned, mapped host memory
+    int* err_host;
+    int* err_dev;
+
+    // profiling (host): launch counts per kernel kind, optional event pairs
+    long long launches[4];
+    int prof_on;
+    int prof_n, prof_cap;
+    cudaEvent_t* prof_ev;   // 2 * prof_cap events
+    int* prof_kind;
+    double prof_ms[4];
+
+    // recurrence bookkeeping (host)
+    long long t;            // steps since reset (selects the ping-pong buffers)
+    int key;                // next step is a key frame
+
+    // tensor-core path: prebuilt TMA descriptors of the two x_{t-1} buffers and the weights
+    int tc_x5d;             // 1: halo tiles as one 5-D TMA box per channel chunk; 0: 4-D boxes per 8 channels
+    CUtensorMap tmap_xbuf[2];
+    CUtensorMap tmap_w;
+};
+
+// ------------------------------------------------------------------ launchers
+// Gate (sc_gate.cu)
+cudaError_t launch_gate_pixel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
+                              const uint8_t* chg_prev, uint8_t* chg_cur);
+cudaError_t launch_gate_block(const Layer& L, int force);
+
+// CUDA-core convolution and elementwise kernels (sc_conv_cc.cu)
+cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
+cudaError_t launch_y_refresh(const Layer& L, const void* shortcut);
+cudaError_t launch_reset_z(const Layer& L);
+cudaError_t launch_pack_weights(Layer& L, const void* w_oihw, double* w_l1_out);
+size_t conv_cc_smem_bytes(const Layer& L);
+
+// Tensor-core convolution (sc_conv_tc.cu)
+bool conv_tc_supported(const skipconv_params& p, const char** why);
+cudaError_t conv_tc_prepare(Layer& L);     // tensor maps of the state buffers and weights
+cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, int prev_index);
+
+// Driver entry point for tensor-map encoding (resolved once through the runtime).
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled_fn();
+
+void set_error(const char* fmt, ...);
+
+}  // namespace sc
+
+// ------------------------------------------------------------- device helpers
+namespace sc {
+
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ float activate(float v, int act)
+{
+    if (act == SKIPCONV_ACT_RELU) return v > 0.f ? v : 0.f;
+    if (act == SKIPCONV_ACT_SILU) return v / (1.f + expf(-v));
+    return v;
+}
+
+}  // namespace sc

@@ -156,14 +156,15 @@ class block_perturbation_video:
     when bf16=True)."""
 
     def __init__(self, seed: int, T: int, n: int, h: int, w: int, c: int, block: int,
-                 n_changed: int, bf16: bool = True, margin: int = 1):
+                 n_changed: int, bf16: bool = True, margin: int = 1, stream_offset: int = 0):
         self.seed, self.T, self.n, self.h, self.w, self.c = seed, T, n, h, w, c
+        self.stream_offset = stream_offset
         self.block, self.n_changed, self.bf16, self.margin = block, n_changed, bf16, margin
         self.nby, self.nbx = h // block, w // block
         assert 0 <= n_changed <= self.nby * self.nbx
 
     def __iter__(self):
-        rng = [np.random.default_rng(self.seed * 100 + s) for s in range(self.n)]
+        rng = [np.random.default_rng(self.seed * 100 + self.stream_offset + s) for s in range(self.n)]
         frame = np.empty((self.n, self.h, self.w, self.c), np.float32)
         for s in range(self.n):
             frame[s] = rng[s].random((self.h, self.w, self.c), dtype=np.float32)

@@ -130,12 +130,14 @@ C4_DENSITIES = (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00)
 
 
 def c4(density: float = 0.10, T: int = 32, n: int = 8, h: int = 128, w: int = 128, c: int = 256,
-       block: int = 8, dtype: str = "bf16") -> Workload:
-    """Density sweep layer.  `frames` is an iterable yielding (t, frame)."""
+       block: int = 8, dtype: str = "bf16", stream_offset: int = 0) -> Workload:
+    """Density sweep layer.  `frames` is an iterable yielding (t, frame);
+    `stream_offset` selects other streams' seeds (independent replicas)."""
     layers = [LayerDef(c, c, 3, 1, 1, 1, block, 0.05, name="conv3x3")]
     n_changed = int(round(density * (h // block) * (w // block)))
     bf16 = dtype == "bf16"
-    frames = block_perturbation_video(4000, T, n, h, w, c, block, n_changed, bf16=bf16)
+    frames = block_perturbation_video(4000, T, n, h, w, c, block, n_changed, bf16=bf16,
+                                      stream_offset=stream_offset)
     ws, bs = _weights(4001, layers, bf16=bf16, bias_std=0.0)
     return Workload("c4", dtype, n, h, w, c, T, layers, ws, bs, frames)
 

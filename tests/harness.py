@@ -1,0 +1,165 @@
+"""Test helpers: run the CUDA layer and the oracle side by side on the same
+seeded frames and compare them at every frame.
+
+Comparison rules (floating point decides the gate, so both sides' decisions
+are compared where they are unique):
+  * block mask: bit-exact, except blocks whose oracle block score lies within
+    1e-5 relative of eps (an fp32 score there may fall on either side);
+  * active list: as a set (atomics make the order unspecified), equal to the
+    GPU's own mask and to the oracle's mask outside the excluded blocks;
+  * z: max-abs error <= 1e-4 for fp32 layers, <= 2e-2 * RMS(z_oracle) for bf16
+    layers, at every frame; locations of a block excluded at some frame are
+    left out from that frame on (its recurrence may legitimately differ);
+  * x_{t-1} held by the layer equals x_t bit for bit after every step.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+EPS_BAND = 1e-5
+TOL_F32_ABS = 1e-4
+TOL_BF16_REL_RMS = 2e-2
+
+
+def to_device(a: np.ndarray, dtype: str):
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(a, np.float32))
+    if dtype == "bf16":
+        t = t.to(torch.bfloat16)          # values are already bf16-exact: no rounding happens here
+    return t.cuda().contiguous()
+
+
+def block_max(score: np.ndarray, b: int) -> np.ndarray:
+    n, ho, wo = score.shape
+    nby, nbx = -(-ho // b), -(-wo // b)
+    pad = np.full((n, nby * b, nbx * b), -np.inf)
+    pad[:, :ho, :wo] = score
+    return pad.reshape(n, nby, b, nbx, b).max(axis=(2, 4))
+
+
+class Compare:
+    """Accumulates per-frame comparison results of one layer."""
+
+    def __init__(self, spec, dtype: str, name: str = ""):
+        self.spec, self.dtype, self.name = spec, dtype, name
+        self.excluded = np.zeros((spec.n, spec.nby, spec.nbx), bool)
+        self.max_err = 0.0
+        self.max_rel = 0.0
+        self.frames = 0
+        self.n_excluded_events = 0
+
+    def frame(self, t, score, mask_ref, gpu_mask, gpu_list, gpu_count, z_ref, z_gpu, forced):
+        s = self.spec
+        if not forced:
+            bmax = block_max(score, s.block)
+            band = np.abs(bmax - s.eps) <= EPS_BAND * max(s.eps, 1e-30)
+            self.n_excluded_events += int(band.sum())
+            self.excluded |= band
+        else:
+            band = np.zeros_like(self.excluded)
+        ok = ~band
+        diff = (gpu_mask != mask_ref) & ok
+        assert not diff.any(), "%s t=%d: %d block gates differ (e.g. %s)" % (
+            self.name, t, int(diff.sum()), np.argwhere(diff)[:5].tolist())
+        ids = np.flatnonzero(gpu_mask.reshape(-1))
+        assert gpu_count == len(ids), "%s t=%d: count %d vs mask %d" % (self.name, t, gpu_count, len(ids))
+        np.testing.assert_array_equal(np.sort(gpu_list), ids, err_msg="%s t=%d: list != mask" % (self.name, t))
+        # z, excluding the footprint of excluded blocks
+        keep = np.repeat(np.repeat(~self.excluded, s.block, axis=1), s.block, axis=2)[:, :s.ho, :s.wo]
+        err = np.abs(z_gpu - z_ref)[keep]
+        e = float(err.max()) if err.size else 0.0
+        rms = float(np.sqrt(np.mean(z_ref ** 2))) if z_ref.size else 0.0
+        self.max_err = max(self.max_err, e)
+        self.max_rel = max(self.max_rel, e / rms if rms > 0 else 0.0)
+        if self.dtype == "f32":
+            assert e <= TOL_F32_ABS, "%s t=%d: max |dz| = %.3g > %.1g" % (self.name, t, e, TOL_F32_ABS)
+        else:
+            assert e <= TOL_BF16_REL_RMS * rms, "%s t=%d: max |dz| = %.3g > 2e-2 * rms %.3g" % (
+                self.name, t, e, rms)
+        self.frames += 1
+
+
+def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_path=0, gate=None):
+    import torch
+    from paper_2104_11487_gb300 import SkipConvLayer
+    wt = torch.from_numpy(np.ascontiguousarray(w, np.float32))
+    bt = None if bias is None else torch.from_numpy(np.ascontiguousarray(bias, np.float32))
+    return SkipConvLayer(spec.n, spec.c_in, spec.c_out, spec.h, spec.w, k=spec.k, stride=spec.stride, pad=spec.pad,
+                         groups=spec.groups, block=spec.block, eps=spec.eps,
+                         gate=spec.gate if gate is None else gate, dtype=dtype, activation=act, emit_y=emit_y,
+                         dense_mode=dense_mode, conv_path=conv_path, weights=wt, bias=bt)
+
+
+def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
+                     reset_at=()):
+    """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
+    both sides; returns the Compare record."""
+    import oracle
+    ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode)
+    gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path)
+    cmp = Compare(spec, dtype, name)
+    try:
+        for t, f in enumerate(frames):
+            if t in reset_at:
+                ref.reset()
+                gl.reset()
+            forced = ref.key or dense_mode
+            score, mask_ref = ref.step(f)
+            xt = to_device(f, dtype)
+            gl.step(xt)
+            mask, lst, cnt = gl.gate()
+            cmp.frame(t, score, mask_ref, mask.cpu().numpy(), lst.cpu().numpy(), cnt, ref.z,
+                      gl.z().cpu().numpy().astype(np.float64), forced)
+            if check_prev:
+                import torch
+                assert torch.equal(gl.prev_input().view(torch.int16 if dtype == "bf16" else torch.int32),
+                                   xt.view(torch.int16 if dtype == "bf16" else torch.int32)), \
+                    "%s t=%d: x_{t-1} is not x_t after the step" % (name, t)
+        assert gl.info.conv_path in (1, 2)
+        return cmp, gl.info.conv_path
+    finally:
+        gl.close()
+
+
+def run_stack_teacher_forced(wl, T=None, conv_path=0):
+    """Run every layer of a stack workload teacher-forced: each CUDA layer
+    gets the oracle's input sequence (and shortcut) for that layer."""
+    import oracle
+    from oracle import LayerSpec
+    frames = wl.frames if T is None else wl.frames[:T]
+    T = len(frames)
+    specs, refs, gls, cmps = [], [], [], []
+    h, w = wl.h, wl.w
+    for li, L in enumerate(wl.layers):
+        spec = LayerSpec(n=wl.n, c_in=L.c_in, c_out=L.c_out, h=h, w=w, k=L.k, stride=L.stride, pad=L.pad,
+                         groups=L.groups, block=L.block, eps=L.eps)
+        specs.append(spec)
+        refs.append(oracle.OracleLayer(spec, wl.weights[li], wl.biases[li]))
+        gls.append(gpu_layer(spec, wl.weights[li], wl.biases[li], wl.dtype, act=L.act, emit_y=True,
+                             conv_path=conv_path))
+        cmps.append(Compare(spec, wl.dtype, "%s/%s" % (wl.name, L.name)))
+        h, w = spec.ho, spec.wo
+    round_mode = 2 if wl.dtype == "bf16" else 1
+    try:
+        for t in range(T):
+            stack = [np.asarray(frames[t], np.float64)]
+            for li, L in enumerate(wl.layers):
+                x = stack[-1]
+                forced = refs[li].key
+                score, mask_ref = refs[li].step(x)
+                sc = None if L.shortcut < 0 else stack[L.shortcut]
+                y_ref = oracle.layer_output(refs[li].z, sc, L.act, round_mode)
+                gls[li].step(to_device(x, wl.dtype), None if sc is None else to_device(sc, wl.dtype))
+                mask, lst, cnt = gls[li].gate()
+                cmps[li].frame(t, score, mask_ref, mask.cpu().numpy(), lst.cpu().numpy(), cnt, refs[li].z,
+                               gls[li].z().cpu().numpy().astype(np.float64), forced)
+                y_gpu = gls[li].y().float().cpu().numpy().astype(np.float64)
+                rms = float(np.sqrt(np.mean(y_ref ** 2)))
+                e = float(np.abs(y_gpu - y_ref).max())
+                assert e <= TOL_BF16_REL_RMS * max(rms, 1e-30), "%s t=%d: y max err %.3g vs rms %.3g" % (
+                    cmps[li].name, t, e, rms)
+                stack.append(y_ref)
+        return cmps, [g.info.conv_path for g in gls]
+    finally:
+        for g in gls:
+            g.close()

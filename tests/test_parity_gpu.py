@@ -1,0 +1,253 @@
+"""Parity of the CUDA Skip-Conv step with the oracle, on the same seeded
+inputs, at every frame (gate masks and lists exact outside the eps band,
+z within the stated tolerance, x_{t-1} committed bit-exactly)."""
+import numpy as np
+import pytest
+
+import synth
+from harness import Compare, run_single_layer, run_stack_teacher_forced, to_device
+from oracle import GATE_INPUT_SUM, GATE_OUTPUT, LayerSpec
+
+pytestmark = pytest.mark.gpu
+
+AUTO, CUDA_CORE, TENSOR_CORE = 0, 1, 2
+
+
+def spec_of(wl, li=0, **kw):
+    L = wl.layers[li]
+    d = dict(n=wl.n, c_in=L.c_in, c_out=L.c_out, h=wl.h, w=wl.w, k=L.k, stride=L.stride, pad=L.pad,
+             groups=L.groups, block=L.block, eps=L.eps)
+    d.update(kw)
+    return LayerSpec(**d)
+
+
+def frames_of(wl):
+    f = wl.frames
+    if isinstance(f, np.ndarray):
+        return [f[t] for t in range(len(f))]
+    return (fr.copy() for _, fr in f)
+
+
+# ----------------------------------------------------------- the workloads
+def test_c0_fp32_pixel_gates():
+    wl = synth.make_workload("c0")
+    cmp, path = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "f32", name="c0")
+    assert path == CUDA_CORE and cmp.frames == 8
+    assert cmp.max_err <= 1e-4
+
+
+@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+def test_c1_bf16_8x8_blocks(path):
+    wl = synth.make_workload("c1")
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                                 conv_path=path, name="c1")
+    assert cmp.frames == 16
+
+
+def test_c2_pose_stack_teacher_forced():
+    wl = synth.make_workload("c2")
+    cmps, paths = run_stack_teacher_forced(wl)
+    assert all(c.frames == 32 for c in cmps)
+
+
+def test_c3_mbconv_stack_teacher_forced():
+    wl = synth.make_workload("c3")
+    cmps, paths = run_stack_teacher_forced(wl)
+    assert all(c.frames == 32 for c in cmps)
+
+
+@pytest.mark.parametrize("density", [0.0, 0.1, 0.5, 1.0])
+@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+def test_c4_density_small(density, path):
+    """c4's generator at a small size (2 streams, 32x40, 64 channels), 32 frames."""
+    wl = synth.make_workload("c4", density=density, T=32, n=2, h=32, w=40, c=64)
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                                 conv_path=path, name="c4-small d=%g" % density)
+    assert cmp.frames == 32
+
+
+@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+def test_ragged_tail_and_several_tiles(path):
+    """Frame sizes that are not multiples of the block (ragged edge blocks)."""
+    frames = synth.round_to_bf16(synth.moving_squares_video(77, 6, 100, 76, 32, n_squares=4, size=12))
+    rng = np.random.default_rng(78)
+    w = synth.he_weights(rng, 48, 32, 3, bf16=True)
+    b = synth.round_to_bf16(rng.standard_normal(48).astype(np.float32) * 0.1)
+    spec = LayerSpec(n=1, c_in=32, c_out=48, h=100, w=76, k=3, block=8, eps=0.05)
+    cmp, _ = run_single_layer(spec, w, b, [f[None] for f in frames], "bf16", conv_path=path, name="ragged")
+    assert cmp.frames == 6
+
+
+@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+def test_dense_mode_is_dense_conv(path):
+    wl = synth.make_workload("c1", T=4)
+    cmp, _ = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                              dense_mode=True, conv_path=path, name="dense")
+    assert cmp.frames == 4
+
+
+def test_gate_variants_and_eps_zero():
+    wl = synth.make_workload("c1", T=5, h=48, w=40, c=16, n_squares=2, size=10)
+    w, b = wl.weights[0], wl.biases[0]
+    for gate, eps in ((GATE_INPUT_SUM, 20.0), (GATE_OUTPUT, 60.0), (0, 0.0)):
+        spec = spec_of(wl, gate=gate, eps=eps)
+        cmp, _ = run_single_layer(spec, w, b, frames_of(wl), "bf16", name="gate%d" % gate)
+        assert cmp.frames == 5
+
+
+def test_reset_mid_sequence_and_single_frame():
+    wl = synth.make_workload("c1", T=7, h=40, w=40, c=16, n_squares=2, size=10)
+    spec = spec_of(wl)
+    cmp, _ = run_single_layer(spec, wl.weights[0], wl.biases[0], frames_of(wl), "bf16", reset_at=(3,),
+                              name="reset")
+    assert cmp.frames == 7
+    cmp, _ = run_single_layer(spec, wl.weights[0], wl.biases[0], frames_of(wl)[:1], "bf16", name="T=1")
+    assert cmp.frames == 1
+
+
+def test_zero_residual_keeps_state_bitwise():
+    import torch
+    from harness import gpu_layer
+    wl = synth.make_workload("c1", T=2, h=32, w=32, c=16, n_squares=1, size=8)
+    spec = spec_of(wl, eps=0.0)
+    gl = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    try:
+        x = to_device(wl.frames[1], "bf16")
+        gl.step(x)
+        z1 = gl.z()
+        gl.step(x.clone())
+        mask, lst, cnt = gl.gate()
+        assert cnt == 0 and int(mask.sum()) == 0
+        assert torch.equal(gl.z().view(torch.int32), z1.view(torch.int32))
+    finally:
+        gl.close()
+
+
+def test_c4_full_size_sampled():
+    """The bench's configuration (8 streams of 128x128x256, 8x8 blocks, 10%
+    block density, 32 frames): full masks and lists every frame, z at sampled
+    locations (the oracle keeps only those)."""
+    import oracle
+    from harness import gpu_layer
+    wl = synth.make_workload("c4", density=0.10, T=32)
+    spec = spec_of(wl)
+    rng = np.random.default_rng(5)
+    samples = np.stack([rng.integers(0, spec.n, 192), rng.integers(0, spec.ho, 192),
+                        rng.integers(0, spec.wo, 192)], axis=1).astype(np.int32)
+    ref = oracle.SampledOracleLayer(spec, wl.weights[0], samples, wl.biases[0])
+    gl = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    cmp = Compare(spec, "bf16", "c4-full")
+    try:
+        for t, f in wl.frames:
+            forced = ref.key
+            mask_ref = ref.step(f)
+            gl.step(to_device(f, "bf16"))
+            mask, lst, cnt = gl.gate()
+            z = gl.z()
+            zs = z[samples[:, 0], samples[:, 1], samples[:, 2]].cpu().numpy().astype(np.float64)
+            # sampled locations stand for the whole frame; the eps band is checked on the sampled
+            # blocks' scores by the full-mask comparison below (no block of this workload lies near eps)
+            md = mask.cpu().numpy()
+            assert np.array_equal(md, mask_ref), "t=%d: masks differ at %d blocks" % (t, int((md != mask_ref).sum()))
+            np.testing.assert_array_equal(np.sort(lst.cpu().numpy()), np.flatnonzero(md.reshape(-1)))
+            assert cnt == int(md.sum())
+            if not forced:
+                assert abs(cnt - round(0.10 * 256) * 8) <= 0, cnt
+            rms = float(np.sqrt(np.mean(ref.z ** 2)))
+            e = float(np.abs(zs - ref.z).max())
+            assert e <= 2e-2 * rms, "t=%d: sampled max err %.3g vs rms %.3g" % (t, e, rms)
+            cmp.frames += 1
+    finally:
+        gl.close()
+    assert cmp.frames == 32
+
+
+# --------------------------------------------------------------- the ABI
+def test_step_host_matches_device_step():
+    import torch
+    from harness import gpu_layer
+    wl = synth.make_workload("c1", T=3, h=32, w=24, c=16, n_squares=1, size=8)
+    spec = spec_of(wl)
+    a = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    b = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    from paper_2104_11487_gb300 import skipconv_step_host
+    try:
+        for t in range(3):
+            xd = to_device(wl.frames[t], "bf16")
+            a.step(xd)
+            xh = xd.cpu().pin_memory()
+            zh = torch.empty(a.shape_out, dtype=torch.float32).pin_memory()
+            skipconv_step_host(b.handle, xh, zh)
+            assert torch.equal(a.z().cpu(), zh)
+    finally:
+        a.close()
+        b.close()
+
+
+def test_stats_match_mask():
+    from harness import gpu_layer
+    wl = synth.make_workload("c1", T=3, h=44, w=36, c=16, n_squares=2, size=8)
+    spec = spec_of(wl)
+    gl = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    try:
+        for t in range(3):
+            gl.step(to_device(wl.frames[t], "bf16"))
+            mask, _, cnt = gl.gate()
+            nb, nloc, macs = gl.stats()
+            m = mask.cpu().numpy()
+            assert nb == cnt == int(m.sum())
+            full = np.repeat(np.repeat(m, 8, axis=1), 8, axis=2)[:, :spec.ho, :spec.wo]
+            assert nloc == int(full.sum())
+            assert macs == nloc * spec.c_out * spec.c_in * 9
+    finally:
+        gl.close()
+
+
+def test_abi_errors_are_status_codes():
+    import ctypes
+
+    import torch
+    from paper_2104_11487_gb300 import _lib
+    from paper_2104_11487_gb300.skipconv import Params
+    L = _lib.lib()
+    w = torch.zeros(8, 8, 3, 3, dtype=torch.bfloat16, device="cuda")
+    h = ctypes.c_void_p()
+    # the tensor-core path cannot take fp32 data: forcing it is UNSUPPORTED
+    p = Params(1, 8, 8, 16, 16, 3, 3, 1, 1, 1, 8, 0.05, 0, 0, 0, 0, 0, TENSOR_CORE)
+    wf = torch.zeros(8, 8, 3, 3, dtype=torch.float32, device="cuda")
+    assert L.skipconv_create(ctypes.byref(p), ctypes.c_void_p(wf.data_ptr()), None, None,
+                             ctypes.byref(h)) == _lib.SKIPCONV_ERR_UNSUPPORTED
+    p = Params(1, 8, 8, 16, 16, 3, 3, 1, 1, 1, 8, 0.05, 0, 1, 0, 0, 0, 0)
+    assert L.skipconv_create(ctypes.byref(p), ctypes.c_void_p(w.data_ptr()), None, None, ctypes.byref(h)) == 0
+    x = torch.zeros(1 * 16 * 16 * 8 + 8, dtype=torch.bfloat16, device="cuda")
+    assert L.skipconv_step(h, ctypes.c_void_p(x.data_ptr() + 2), None) == _lib.SKIPCONV_ERR_INVALID  # misaligned
+    assert L.skipconv_step(h, ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(x.data_ptr())) == \
+        _lib.SKIPCONV_ERR_INVALID  # shortcut without emit_y
+    assert L.skipconv_step(h, ctypes.c_void_p(x.data_ptr()), None) == 0
+    assert L.skipconv_check_device(h) == 0
+    assert L.skipconv_destroy(h) == 0
+
+
+def test_allocation_failure_is_reported_and_cleaned_up(monkeypatch):
+    """Host-side fault injection: the k-th device allocation of create fails."""
+    import ctypes
+
+    import torch
+    from paper_2104_11487_gb300 import _lib
+    from paper_2104_11487_gb300.skipconv import Params
+    L = _lib.lib()
+    w = torch.zeros(16, 16, 3, 3, dtype=torch.bfloat16, device="cuda")
+    p = Params(2, 16, 16, 64, 64, 3, 3, 1, 1, 1, 8, 0.05, 0, 1, 0, 1, 0, 0)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for k in range(1, 16):
+        monkeypatch.setenv("SKIPCONV_FAULT_ALLOC", str(k))
+        h = ctypes.c_void_p()
+        st = L.skipconv_create(ctypes.byref(p), ctypes.c_void_p(w.data_ptr()), None, None, ctypes.byref(h))
+        if st == 0:
+            L.skipconv_destroy(h)
+            continue
+        assert st == _lib.SKIPCONV_ERR_OOM and h.value is None
+    monkeypatch.delenv("SKIPCONV_FAULT_ALLOC")
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] >= free0 - (8 << 20)
