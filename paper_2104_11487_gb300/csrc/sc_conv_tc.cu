@@ -19,8 +19,11 @@
 // with tcgen05.ld and add it into z in place (the scatter-accumulate of
 // Eq. 3), optionally writing y = act(z).
 //
-// Warp roles: 0-3 epilogue, 4-7 residual, 8 TMA producer, 9 MMA issuer.
+// Warp roles: 0-3 epilogue, 4-7 residual, 8 weight-tile producer, 9 MMA issuer,
+// 10 halo-tile producer (separate so that the weight stream never waits on
+// the halo ring, and vice versa).
 #include <math.h>
+#include <stdlib.h>
 
 #include "sc_internal.h"
 #include "sc_ptx.cuh"
@@ -33,9 +36,10 @@ constexpr int TC_N = 64;
 constexpr int TC_CK = 64;          // input channels per K chunk
 constexpr int TC_ASTAGES = 8;
 constexpr int TC_XSTAGES = 2;
-constexpr int TC_THREADS = 320;
+constexpr int TC_THREADS = 352;
 constexpr int TC_ABYTES = TC_M * TC_CK * 2;  // 16 KiB weight tile
 constexpr uint32_t TC_TMEM_COLS = 2 * TC_N;
+constexpr int TC_ZBYTES = TC_N * TC_M * 4;   // fp32 staging tile of one unit's result
 constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;
 
 struct TcArgs {
@@ -48,6 +52,7 @@ struct TcArgs {
     int H, W, Ho, Wo, Co, KH, KW, pad, nby, nbx;
     int n_ct, n_chunks, HH, WW, taps, ci_pad;
     int x5d;
+    int z_tma;   // 1: z += D through a TMA reduce-add (no y); 0: load, add, store (and y)
 };
 
 struct Bars {
@@ -59,11 +64,13 @@ struct Bars {
     int abort;
 };
 
+// Bytes of one halo tile (one tensor, one 64-channel chunk) in shared memory.
 __host__ __device__ inline int x_tile_bytes(int HH, int WW) { return 8 * HH * WW * 16; }
 
 size_t tc_smem_bytes(int HH, int WW)
 {
-    return 1024 + (size_t)TC_ASTAGES * TC_ABYTES + (size_t)TC_XSTAGES * 2 * x_tile_bytes(HH, WW) + sizeof(Bars);
+    return 1024 + (size_t)TC_ASTAGES * TC_ABYTES + (size_t)TC_XSTAGES * 2 * x_tile_bytes(HH, WW) + TC_ZBYTES +
+           sizeof(Bars);
 }
 
 __device__ __forceinline__ void decode_unit(const TcArgs& a, int u, int& n, int& by, int& bx, int& ct)
@@ -93,14 +100,15 @@ __device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant__ CUtensorMap tm_xp,
-               const __grid_constant__ CUtensorMap tm_w, const TcArgs a)
+               const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_z, const TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int XB = x_tile_bytes(a.HH, a.WW);
     uint8_t* sA = smem;
     uint8_t* sX = smem + TC_ASTAGES * TC_ABYTES;
-    Bars* bars = (Bars*)(sX + TC_XSTAGES * 2 * XB);
+    float* sZ = (float*)(sX + TC_XSTAGES * 2 * XB);
+    Bars* bars = (Bars*)((uint8_t*)sZ + TC_ZBYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int units = a.counters[0] * a.n_ct;
     if ((int)blockIdx.x >= units) return;
@@ -133,64 +141,65 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
     const uint32_t tmem = bars->tmem_base;
     volatile int* abort = &bars->abort;
 
-    if (warp == 8) {
-        // ------------------------------------------------ TMA producer
+    if (warp == 8 || warp == 10) {
+        // ------------------------------------------------ TMA producers
         if (lane == 0) {
-            ptx::prefetch_tmap(&tm_xt);
-            ptx::prefetch_tmap(&tm_xp);
-            ptx::prefetch_tmap(&tm_w);
-            int xs = 0, as = 0;
-            uint32_t xph = 0, aph = 0;
-            uint32_t x_issue_ph[TC_XSTAGES] = {0, 0}, a_issue_ph[TC_ASTAGES] = {};
-            uint32_t x_issued = 0, a_issued = 0;  // bit per stage: a load was issued there
+            const bool halo = warp == 10;
+            ptx::prefetch_tmap(halo ? &tm_xt : &tm_w);
+            if (halo) ptx::prefetch_tmap(&tm_xp);
+            int st = 0;
+            uint32_t ph = 0;
+            uint32_t issue_ph[TC_ASTAGES] = {};
+            uint32_t issued = 0;  // bit per stage: a load was issued there
             bool ok = true;
             for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
                 int n, by, bx, ct;
                 decode_unit(a, u, n, by, bx, ct);
                 const int y0 = by * 8 - a.pad, x0 = bx * 8 - a.pad;
                 for (int c = 0; c < a.n_chunks && ok; ++c) {
-                    const uint32_t xf = ptx::smem_u32(&bars->x_full[xs]);
-                    if (!(ok = ptx::mbar_wait(ptx::smem_u32(&bars->x_empty[xs]), xph ^ 1, abort, a.err, WAIT_LIMIT_NS)))
-                        break;
-                    ptx::mbar_arrive_expect_tx(xf, 2 * XB);
-                    const uint32_t dst = ptx::smem_u32(sX + xs * 2 * XB);
-                    if (a.x5d) {
-                        ptx::tma_load_5d(dst, &tm_xt, xf, 0, x0, y0, c * 8, n);
-                        ptx::tma_load_5d(dst + XB, &tm_xp, xf, 0, x0, y0, c * 8, n);
-                    } else {
-                        const int gb = a.HH * a.WW * 16;
-                        for (int g = 0; g < 8; ++g) {
-                            ptx::tma_load_4d(dst + g * gb, &tm_xt, xf, (c * 8 + g) * 8, x0, y0, n);
-                            ptx::tma_load_4d(dst + XB + g * gb, &tm_xp, xf, (c * 8 + g) * 8, x0, y0, n);
-                        }
-                    }
-                    x_issue_ph[xs] = xph;
-                    x_issued |= 1u << xs;
-                    if (++xs == TC_XSTAGES) { xs = 0; xph ^= 1; }
-                    for (int t = 0; t < a.taps; ++t) {
-                        const uint32_t af = ptx::smem_u32(&bars->a_full[as]);
-                        if (!(ok = ptx::mbar_wait(ptx::smem_u32(&bars->a_empty[as]), aph ^ 1, abort, a.err,
+                    if (halo) {
+                        const uint32_t xf = ptx::smem_u32(&bars->x_full[st]);
+                        if (!(ok = ptx::mbar_wait(ptx::smem_u32(&bars->x_empty[st]), ph ^ 1, abort, a.err,
                                                   WAIT_LIMIT_NS)))
                             break;
-                        ptx::mbar_arrive_expect_tx(af, TC_ABYTES);
-                        ptx::tma_load_2d(ptx::smem_u32(sA + as * TC_ABYTES), &tm_w, af, t * a.ci_pad + c * TC_CK,
-                                         ct * TC_M);
-                        a_issue_ph[as] = aph;
-                        a_issued |= 1u << as;
-                        if (++as == TC_ASTAGES) { as = 0; aph ^= 1; }
+                        ptx::mbar_arrive_expect_tx(xf, 2 * XB);
+                        const uint32_t dst = ptx::smem_u32(sX + st * 2 * XB);
+                        if (a.x5d) {
+                            ptx::tma_load_5d(dst, &tm_xt, xf, 0, x0, y0, c * 8, n);
+                            ptx::tma_load_5d(dst + XB, &tm_xp, xf, 0, x0, y0, c * 8, n);
+                        } else {
+                            const int gb = a.HH * a.WW * 16;
+                            for (int g = 0; g < 8; ++g) {
+                                ptx::tma_load_4d(dst + g * gb, &tm_xt, xf, (c * 8 + g) * 8, x0, y0, n);
+                                ptx::tma_load_4d(dst + XB + g * gb, &tm_xp, xf, (c * 8 + g) * 8, x0, y0, n);
+                            }
+                        }
+                        issue_ph[st] = ph;
+                        issued |= 1u << st;
+                        if (++st == TC_XSTAGES) { st = 0; ph ^= 1; }
+                    } else {
+                        for (int t = 0; t < a.taps; ++t) {
+                            const uint32_t af = ptx::smem_u32(&bars->a_full[st]);
+                            if (!(ok = ptx::mbar_wait(ptx::smem_u32(&bars->a_empty[st]), ph ^ 1, abort, a.err,
+                                                      WAIT_LIMIT_NS)))
+                                break;
+                            ptx::mbar_arrive_expect_tx(af, TC_ABYTES);
+                            ptx::tma_load_2d(ptx::smem_u32(sA + st * TC_ABYTES), &tm_w, af,
+                                             t * a.ci_pad + c * TC_CK, ct * TC_M);
+                            issue_ph[st] = ph;
+                            issued |= 1u << st;
+                            if (++st == TC_ASTAGES) { st = 0; ph ^= 1; }
+                        }
                     }
                 }
             }
             if (!ok) {
                 // let every copy this thread started land before the CTA exits
-                for (int s = 0; s < TC_XSTAGES; ++s)
-                    if (x_issued & (1u << s))
-                        ptx::mbar_wait(ptx::smem_u32(&bars->x_full[s]), x_issue_ph[s], nullptr, nullptr,
-                                       WAIT_LIMIT_NS);
-                for (int s = 0; s < TC_ASTAGES; ++s)
-                    if (a_issued & (1u << s))
-                        ptx::mbar_wait(ptx::smem_u32(&bars->a_full[s]), a_issue_ph[s], nullptr, nullptr,
-                                       WAIT_LIMIT_NS);
+                const int nst = halo ? TC_XSTAGES : TC_ASTAGES;
+                for (int s2 = 0; s2 < nst; ++s2)
+                    if (issued & (1u << s2))
+                        ptx::mbar_wait(ptx::smem_u32(halo ? &bars->x_full[s2] : &bars->a_full[s2]), issue_ph[s2],
+                                       nullptr, nullptr, WAIT_LIMIT_NS);
             }
         }
     } else if (warp == 9) {
@@ -266,6 +275,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
         }
     } else {
         // ------------------------------------------- epilogue: z += D
+        const int tid = threadIdx.x;  // 0..127
         int acc = 0;
         uint32_t accph = 0;
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
@@ -282,23 +292,50 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&bars->acc_empty[acc]));
             if (++acc == 2) { acc = 0; accph ^= 1; }
-            const int co = ct * TC_M + warp * 32 + lane;
-            if (co < a.Co) {
-                const bool full = (by * 8 + 8 <= a.Ho) && (bx * 8 + 8 <= a.Wo);
-                float* zb = a.z + ((size_t)n * a.Ho * a.Wo) * a.Co + co;
+            const int col = warp * 32 + lane;  // output channel within the tile
+            if (a.z_tma) {
+                // stage D as [pixel][channel] fp32 and add it into z at L2
+                if (tid == 0) ptx::bulk_wait_group_read0();
+                ptx::named_bar_sync(1, 128);
 #pragma unroll
-                for (int p = 0; p < 64; ++p) {
-                    const int oy = by * 8 + (p >> 3), ox = bx * 8 + (p & 7);
-                    if (full || (oy < a.Ho && ox < a.Wo)) {
-                        const size_t off = ((size_t)oy * a.Wo + ox) * a.Co;
-                        const float dv = __uint_as_float(p < 32 ? r0[p] : r1[p - 32]);
-                        const float v = zb[off] + dv;
-                        zb[off] = v;
-                        if (a.y) a.y[(size_t)n * a.Ho * a.Wo * a.Co + off + co] = __float2bfloat16_rn(activate(v, a.act));
+                for (int p = 0; p < 32; ++p) {
+                    sZ[p * TC_M + col] = __uint_as_float(r0[p]);
+                    sZ[(p + 32) * TC_M + col] = __uint_as_float(r1[p]);
+                }
+                ptx::fence_proxy_async_smem();
+                ptx::named_bar_sync(1, 128);
+                if (tid == 0) {
+                    ptx::tma_reduce_add_4d(&tm_z, ptx::smem_u32(sZ), ct * TC_M, bx * 8, by * 8, n);
+                    ptx::bulk_commit_group();
+                }
+            } else {
+                const int co = ct * TC_M + col;
+                if (co < a.Co) {
+                    float* zb = a.z + ((size_t)n * a.Ho * a.Wo) * a.Co + co;
+                    __nv_bfloat16* yb = a.y ? a.y + ((size_t)n * a.Ho * a.Wo) * a.Co + co : nullptr;
+                    // one output row (8 pixels) at a time: 8 loads in flight, then 8 stores
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int oy = by * 8 + i;
+                        if (oy >= a.Ho) break;
+                        float* zr = zb + ((size_t)oy * a.Wo + bx * 8) * a.Co;
+                        float zv[8];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) zv[j] = (bx * 8 + j < a.Wo) ? zr[(size_t)j * a.Co] : 0.f;
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            if (bx * 8 + j < a.Wo) {
+                                const int q = i * 8 + j;
+                                const float v = zv[j] + __uint_as_float(q < 32 ? r0[q & 31] : r1[q & 31]);
+                                zr[(size_t)j * a.Co] = v;
+                                if (yb) yb[((size_t)oy * a.Wo + bx * 8 + j) * a.Co] = __float2bfloat16_rn(activate(v, a.act));
+                            }
+                        }
                     }
                 }
             }
         }
+        if (a.z_tma && tid == 0) ptx::bulk_wait_group0();
     }
 
     ptx::tc_fence_before();
@@ -336,6 +373,20 @@ bool encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d)
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     }
     return r == CUDA_SUCCESS;
+}
+
+bool encode_z_map(CUtensorMap* m, const Layer& L)
+{
+    EncodeTiledFn enc = encode_tiled_fn();
+    if (!enc || L.p.c_out % 4) return false;
+    const cuuint64_t Co = L.p.c_out, Wo = L.wo, Ho = L.ho, N = L.p.n_streams;
+    cuuint64_t dims[4] = {Co, Wo, Ho, N};
+    cuuint64_t strides[3] = {Co * 4, Wo * Co * 4, Ho * Wo * Co * 4};
+    cuuint32_t box[4] = {TC_M, 8, 8, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, L.z, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -379,6 +430,7 @@ cudaError_t conv_tc_prepare(Layer& L)
         set_error("tensor map of the weights rejected (%d)", (int)r);
         return cudaErrorInvalidValue;
     }
+    L.tc_z_tma = encode_z_map(&L.tmap_z, L) ? 1 : 0;
     const int HH = 8 + L.p.k_h - 1, WW = 8 + L.p.k_w - 1;
     return cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)tc_smem_bytes(HH, WW));
@@ -416,10 +468,11 @@ cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, 
     a.taps = L.p.k_h * L.p.k_w;
     a.ci_pad = L.ci_pad;
     a.x5d = L.tc_x5d;
+    a.z_tma = (L.y == nullptr && L.tc_z_tma) ? 1 : 0;
     const long long max_units = (long long)L.p.n_streams * L.nby * L.nbx * a.n_ct;
     const int grid = (int)(max_units < L.num_sms ? max_units : L.num_sms);
     conv_tc_kernel<<<grid, TC_THREADS, tc_smem_bytes(a.HH, a.WW), L.stream>>>(tm_xt, L.tmap_xbuf[prev_index],
-                                                                              L.tmap_w, a);
+                                                                              L.tmap_w, L.tmap_z, a);
     return cudaGetLastError();
 }
 

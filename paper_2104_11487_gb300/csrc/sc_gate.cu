@@ -48,8 +48,10 @@ __device__ __forceinline__ unsigned bits_differ(const uint4& a, const uint4& b)
 }
 
 // 16-byte vector path: a pixel's channels are `cpp` 16-byte chunks, handled
-// by a group of G = 2^log2g lanes (each lane up to PER chunks).
-template <typename T, int PER>
+// by a group of G = 2^log2g lanes (each lane up to PER chunks).  Each warp
+// iteration covers U consecutive groups of pixels so that 2*U*PER loads per
+// lane are in flight before the first reduction.
+template <typename T, int PER, int U>
 __global__ void __launch_bounds__(256) gate_pixel_vec_kernel(
     const uint4* __restrict__ xt, const uint4* __restrict__ xp, uint4* __restrict__ xn,
     const uint8_t* __restrict__ chg_prev, uint8_t* __restrict__ chg_cur, float* __restrict__ pix_l1,
@@ -62,40 +64,52 @@ __global__ void __launch_bounds__(256) gate_pixel_vec_kernel(
     const int gpw = 32 >> log2g;
     const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    for (long long base = warp * gpw; base < n_pix; base += nwarps * gpw) {
-        const long long pix = base + (lane >> log2g);
-        const bool valid = pix < n_pix;
-        uint4 a[PER];
-        float s = 0.f;
-        unsigned diff = 0;
+    for (long long base = warp * gpw * U; base < n_pix; base += nwarps * gpw * U) {
+        uint4 a[U][PER], b[U][PER];
 #pragma unroll
-        for (int k = 0; k < PER; ++k) {
-            const int c = sub + k * G;
-            if (valid && c < cpp) {
-                a[k] = __ldg(xt + pix * cpp + c);
-                const uint4 b = __ldg(xp + pix * cpp + c);
-                s += l1_diff(a[k], b, (T*)nullptr);
-                diff |= bits_differ(a[k], b);
-            }
-        }
+        for (int v = 0; v < U; ++v) {
+            const long long pix = base + v * gpw + (lane >> log2g);
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-            if (off < G) {
-                s += __shfl_xor_sync(0xffffffffu, s, off);
-                diff |= __shfl_xor_sync(0xffffffffu, diff, off);
-            }
-        }
-        if (valid) {
-            if (diff || chg_prev[pix]) {
-#pragma unroll
-                for (int k = 0; k < PER; ++k) {
-                    const int c = sub + k * G;
-                    if (c < cpp) xn[pix * cpp + c] = a[k];
+            for (int k = 0; k < PER; ++k) {
+                const int c = sub + k * G;
+                if (pix < n_pix && c < cpp) {
+                    a[v][k] = __ldg(xt + pix * cpp + c);
+                    b[v][k] = __ldg(xp + pix * cpp + c);
+                } else {
+                    a[v][k] = make_uint4(0, 0, 0, 0);
+                    b[v][k] = make_uint4(0, 0, 0, 0);
                 }
             }
-            if (sub == 0) {
-                pix_l1[pix] = s;
-                chg_cur[pix] = diff ? 1 : 0;
+        }
+#pragma unroll
+        for (int v = 0; v < U; ++v) {
+            const long long pix = base + v * gpw + (lane >> log2g);
+            float s = 0.f;
+            unsigned diff = 0;
+#pragma unroll
+            for (int k = 0; k < PER; ++k) {
+                s += l1_diff(a[v][k], b[v][k], (T*)nullptr);
+                diff |= bits_differ(a[v][k], b[v][k]);
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                if (off < G) {
+                    s += __shfl_xor_sync(0xffffffffu, s, off);
+                    diff |= __shfl_xor_sync(0xffffffffu, diff, off);
+                }
+            }
+            if (pix < n_pix) {
+                if (diff || chg_prev[pix]) {
+#pragma unroll
+                    for (int k = 0; k < PER; ++k) {
+                        const int c = sub + k * G;
+                        if (c < cpp) xn[pix * cpp + c] = a[v][k];
+                    }
+                }
+                if (sub == 0) {
+                    pix_l1[pix] = s;
+                    chg_cur[pix] = diff ? 1 : 0;
+                }
             }
         }
     }
@@ -159,15 +173,22 @@ __global__ void __launch_bounds__(256) gate_pixel_elem_kernel(
     }
 }
 
+// One warp per gate block.  The block's input footprint of per-pixel norms
+// (FH x FW with FH = (b-1)*stride + k_h) is staged in shared memory with one
+// round of coalesced loads; each lane then box-sums the supports of its
+// output locations from shared memory.  When the footprint is too large for
+// the staging area (stage == 0) the sums read global memory directly.
 __global__ void __launch_bounds__(256) gate_block_kernel(
     const float* __restrict__ pix_l1, uint8_t* __restrict__ mask, int32_t* __restrict__ list,
     int32_t* __restrict__ counters, int n, int H, int W, int Ho, int Wo, int KH, int KW, int stride, int pad,
-    int b, int nby, int nbx, float thr, int force)
+    int b, int nby, int nbx, float thr, int force, int stage)
 {
+    extern __shared__ float foot[];  // [8 warps][FH*FW] when staging
     __shared__ int flags[8];
     const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long nblocks = (long long)n * nby * nbx;
     const long long blk = (long long)blockIdx.x * 8 + wid;
+    const int FH = (b - 1) * stride + KH, FW = (b - 1) * stride + KW;
     int open = 0;
     if (blk < nblocks) {
         if (force) {
@@ -179,19 +200,29 @@ __global__ void __launch_bounds__(256) gate_block_kernel(
             const int nn = (int)(rest / nby);
             const float* P = pix_l1 + (size_t)nn * H * W;
             const int bh = min(b, Ho - by * b), bw = min(b, Wo - bx * b);
+            const int fy0 = by * b * stride - pad, fx0 = bx * b * stride - pad;
+            float* F = foot + wid * FH * FW;
+            if (stage) {
+                for (int q = lane; q < FH * FW; q += 32) {
+                    const int yy = fy0 + q / FW, xx = fx0 + q % FW;
+                    F[q] = (yy >= 0 && yy < H && xx >= 0 && xx < W) ? __ldg(P + (size_t)yy * W + xx) : 0.f;
+                }
+                __syncwarp();
+            }
             float best = -1.f;
             for (int q = lane; q < bh * bw; q += 32) {
-                const int i = by * b + q / bw, j = bx * b + q % bw;
+                const int i = q / bw, j = q % bw;  // within the block
                 float S = 0.f;
-                for (int kh = 0; kh < KH; ++kh) {
-                    const int yy = i * stride + kh - pad;
-                    if (yy < 0 || yy >= H) continue;
+                for (int kh = 0; kh < KH; ++kh)
                     for (int kw = 0; kw < KW; ++kw) {
-                        const int xx = j * stride + kw - pad;
-                        if (xx < 0 || xx >= W) continue;
-                        S += __ldg(P + (size_t)yy * W + xx);
+                        const int fy = i * stride + kh, fx = j * stride + kw;
+                        if (stage) {
+                            S += F[fy * FW + fx];
+                        } else {
+                            const int yy = fy0 + fy, xx = fx0 + fx;
+                            if (yy >= 0 && yy < H && xx >= 0 && xx < W) S += __ldg(P + (size_t)yy * W + xx);
+                        }
                     }
-                }
                 best = fmaxf(best, S);
             }
 #pragma unroll
@@ -235,11 +266,11 @@ cudaError_t launch_pixel_typed(const Layer& L, const void* x_t, const void* x_pr
         const uint4* b = (const uint4*)x_prev;
         uint4* c = (uint4*)x_next;
         if (per == 1)
-            gate_pixel_vec_kernel<T, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
+            gate_pixel_vec_kernel<T, 1, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
         else if (per == 2)
-            gate_pixel_vec_kernel<T, 2><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
+            gate_pixel_vec_kernel<T, 2, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
         else if (per <= 4)
-            gate_pixel_vec_kernel<T, 4><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
+            gate_pixel_vec_kernel<T, 4, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
         else
             return cudaErrorInvalidValue;
     } else {
@@ -284,9 +315,12 @@ cudaError_t launch_gate_block(const Layer& L, int force)
 {
     const long long nblocks = (long long)L.p.n_streams * L.nby * L.nbx;
     const int grid = (int)((nblocks + 7) / 8);
-    gate_block_kernel<<<grid, 256, 0, L.stream>>>(L.pix_l1, L.mask, L.list, L.counters, L.p.n_streams, L.p.h,
-                                                  L.p.w, L.ho, L.wo, L.p.k_h, L.p.k_w, L.p.stride, L.p.pad,
-                                                  L.p.block, L.nby, L.nbx, L.gate_thr, force);
+    const int FH = (L.p.block - 1) * L.p.stride + L.p.k_h, FW = (L.p.block - 1) * L.p.stride + L.p.k_w;
+    const size_t foot = (size_t)8 * FH * FW * sizeof(float);
+    const int stage = foot <= 40 * 1024 ? 1 : 0;
+    gate_block_kernel<<<grid, 256, stage ? foot : 0, L.stream>>>(
+        L.pix_l1, L.mask, L.list, L.counters, L.p.n_streams, L.p.h, L.p.w, L.ho, L.wo, L.p.k_h, L.p.k_w,
+        L.p.stride, L.p.pad, L.p.block, L.nby, L.nbx, L.gate_thr, force, stage);
     return cudaGetLastError();
 }
 

@@ -61,6 +61,8 @@ struct Layer {
     int tc_x5d;             // 1: halo tiles as one 5-D TMA box per channel chunk; 0: 4-D boxes per 8 channels
     CUtensorMap tmap_xbuf[2];
     CUtensorMap tmap_w;
+    int tc_z_tma;           // 1: the z tensor map below is valid (c_out multiple of 4)
+    CUtensorMap tmap_z;
 };
 
 // ------------------------------------------------------------------ launchers

@@ -153,11 +153,14 @@ def run_stack_teacher_forced(wl, T=None, conv_path=0):
                 mask, lst, cnt = gls[li].gate()
                 cmps[li].frame(t, score, mask_ref, mask.cpu().numpy(), lst.cpu().numpy(), cnt, refs[li].z,
                                gls[li].z().cpu().numpy().astype(np.float64), forced)
+                # y = round_bf16(act(z [+ shortcut])): the z tolerance, plus one bf16 ulp of the value,
+                # since z values a few fp32 ulps apart may round to neighbouring bf16 values
                 y_gpu = gls[li].y().float().cpu().numpy().astype(np.float64)
                 rms = float(np.sqrt(np.mean(y_ref ** 2)))
-                e = float(np.abs(y_gpu - y_ref).max())
-                assert e <= TOL_BF16_REL_RMS * max(rms, 1e-30), "%s t=%d: y max err %.3g vs rms %.3g" % (
-                    cmps[li].name, t, e, rms)
+                allowed = TOL_BF16_REL_RMS * rms + np.abs(y_ref) * 2.0 ** -7 + 1e-30
+                bad = np.abs(y_gpu - y_ref) > allowed
+                assert not bad.any(), "%s t=%d: %d y values beyond tolerance (max err %.3g, rms %.3g)" % (
+                    cmps[li].name, t, int(bad.sum()), float(np.abs(y_gpu - y_ref).max()), rms)
                 stack.append(y_ref)
         return cmps, [g.info.conv_path for g in gls]
     finally:
