@@ -316,6 +316,10 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
     L.gate_thr = (float)thr;
 
     if (e == cudaSuccess && L.path == SKIPCONV_PATH_TENSOR_CORE) e = conv_tc_prepare(L);
+    if (e == cudaSuccess && L.path == SKIPCONV_PATH_TENSOR_CORE && conv_ws_supported(L)) {
+        e = conv_ws_prepare(L);
+        L.tc_ws = e == cudaSuccess ? 1 : 0;
+    }
     if (e == cudaSuccess) {
         h->L.key = 1;
         st = skipconv_reset_state(h);
@@ -343,6 +347,7 @@ int skipconv_reset_state(skipconv_handle h)
     if (e == cudaSuccess) e = cudaMemsetAsync(L->xbuf[1], 0, xbytes, L->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[0], 0, npix, L->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[1], 0, npix, L->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->counters, 0, 64 * sizeof(int32_t), L->stream);
     if (e == cudaSuccess) e = launch_reset_z(*L);
     if (e == cudaSuccess && L->y) e = cudaMemsetAsync(L->y, 0, (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * L->esize, L->stream);
     if (e != cudaSuccess) return status_of(e);
@@ -364,16 +369,13 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     // xbuf[cur] holds x_{t-1}; xbuf[nxt] holds x_{t-2} and receives x_t.
     // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
     int slot = prof_begin(L, 0);
-    cudaError_t e = launch_gate_pixel(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur]);
+    cudaError_t e = launch_gate(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur],
+                                (L->key || L->p.dense_mode) ? 1 : 0);
     prof_end(L, slot);
     if (e == cudaSuccess) {
-        slot = prof_begin(L, 1);
-        e = launch_gate_block(*L, (L->key || L->p.dense_mode) ? 1 : 0);
-        prof_end(L, slot);
-    }
-    if (e == cudaSuccess) {
         slot = prof_begin(L, 2);
-        if (L->path == SKIPCONV_PATH_TENSOR_CORE) e = launch_conv_tc(*L, x_t, L->xbuf[cur], cur);
+        if (L->path == SKIPCONV_PATH_TENSOR_CORE && L->tc_ws) e = launch_conv_ws(*L, x_t, cur);
+        else if (L->path == SKIPCONV_PATH_TENSOR_CORE) e = launch_conv_tc(*L, x_t, L->xbuf[cur], cur);
         else e = launch_conv_cc(*L, x_t, L->xbuf[cur]);
         prof_end(L, slot);
     }
@@ -459,7 +461,7 @@ int skipconv_get_gate(skipconv_handle h, const uint8_t** block_mask, const int32
     if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
     if (block_mask) *block_mask = L->mask;
     if (active_list) *active_list = L->list;
-    if (active_count) *active_count = L->counters;
+    if (active_count) *active_count = L->counters + ((L->t + 1) & 1);  // slot of the last step (t - 1)
     return SKIPCONV_OK;
 }
 

@@ -135,11 +135,11 @@ cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev)
         auto k = conv_cc_kernel<__nv_bfloat16>;
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         k<<<grid, 256, smem, L.stream>>>((const __nv_bfloat16*)x_t, (const __nv_bfloat16*)x_prev, L.w_cc, L.list,
-                                         L.counters, L.z, (__nv_bfloat16*)L.y, L.p.activation, g);
+                                         step_count(L), L.z, (__nv_bfloat16*)L.y, L.p.activation, g);
     } else {
         auto k = conv_cc_kernel<float>;
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        k<<<grid, 256, smem, L.stream>>>((const float*)x_t, (const float*)x_prev, L.w_cc, L.list, L.counters, L.z,
+        k<<<grid, 256, smem, L.stream>>>((const float*)x_t, (const float*)x_prev, L.w_cc, L.list, step_count(L), L.z,
                                          (float*)L.y, L.p.activation, g);
     }
     return cudaGetLastError();

@@ -27,19 +27,16 @@
 
 #include "sc_internal.h"
 #include "sc_ptx.cuh"
+#include "sc_tc_common.cuh"
 
 namespace sc {
 namespace {
 
-constexpr int TC_M = 128;
-constexpr int TC_N = 64;
-constexpr int TC_CK = 64;          // input channels per K chunk
 constexpr int TC_ASTAGES = 8;
 constexpr int TC_XSTAGES = 2;
 constexpr int TC_THREADS = 352;
 constexpr int TC_ABYTES = TC_M * TC_CK * 2;  // 16 KiB weight tile
 constexpr uint32_t TC_TMEM_COLS = 2 * TC_N;
-constexpr int TC_ZBYTES = TC_N * TC_M * 4;   // fp32 staging tile of one unit's result
 constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;
 
 struct TcArgs {
@@ -64,9 +61,6 @@ struct Bars {
     int abort;
 };
 
-// Bytes of one halo tile (one tensor, one 64-channel chunk) in shared memory.
-__host__ __device__ inline int x_tile_bytes(int HH, int WW) { return 8 * HH * WW * 16; }
-
 size_t tc_smem_bytes(int HH, int WW)
 {
     return 1024 + (size_t)TC_ASTAGES * TC_ABYTES + (size_t)TC_XSTAGES * 2 * x_tile_bytes(HH, WW) + TC_ZBYTES +
@@ -81,21 +75,6 @@ __device__ __forceinline__ void decode_unit(const TcArgs& a, int u, int& n, int&
     bx = id % a.nbx;
     by = (id / a.nbx) % a.nby;
     n = id / (a.nbx * a.nby);
-}
-
-__device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
-{
-    const __nv_bfloat162* a = reinterpret_cast<const __nv_bfloat162*>(&x);
-    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&p);
-    uint4 out;
-    __nv_bfloat162* o = reinterpret_cast<__nv_bfloat162*>(&out);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const float2 fa = __bfloat1622float2(a[k]);
-        const float2 fb = __bfloat1622float2(b[k]);
-        o[k] = __floats2bfloat162_rn(fa.x - fb.x, fa.y - fb.y);
-    }
-    return out;
 }
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
@@ -348,7 +327,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
 }
 
 // ------------------------------------------------------------ tensor maps
-bool encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d)
+}  // namespace
+
+bool tc_encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d)
 {
     EncodeTiledFn enc = encode_tiled_fn();
     if (!enc) return false;
@@ -375,7 +356,7 @@ bool encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d)
     return r == CUDA_SUCCESS;
 }
 
-bool encode_z_map(CUtensorMap* m, const Layer& L)
+bool tc_encode_z_map(CUtensorMap* m, const Layer& L)
 {
     EncodeTiledFn enc = encode_tiled_fn();
     if (!enc || L.p.c_out % 4) return false;
@@ -388,8 +369,6 @@ bool encode_z_map(CUtensorMap* m, const Layer& L)
                CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
-
-}  // namespace
 
 bool conv_tc_supported(const skipconv_params& p, const char** why)
 {
@@ -411,9 +390,9 @@ cudaError_t conv_tc_prepare(Layer& L)
         return cudaErrorNotSupported;
     }
     L.tc_x5d = 1;
-    if (!encode_x_map(&L.tmap_xbuf[0], L.xbuf[0], L, true) || !encode_x_map(&L.tmap_xbuf[1], L.xbuf[1], L, true)) {
+    if (!tc_encode_x_map(&L.tmap_xbuf[0], L.xbuf[0], L, true) || !tc_encode_x_map(&L.tmap_xbuf[1], L.xbuf[1], L, true)) {
         L.tc_x5d = 0;
-        if (!encode_x_map(&L.tmap_xbuf[0], L.xbuf[0], L, false) || !encode_x_map(&L.tmap_xbuf[1], L.xbuf[1], L, false)) {
+        if (!tc_encode_x_map(&L.tmap_xbuf[0], L.xbuf[0], L, false) || !tc_encode_x_map(&L.tmap_xbuf[1], L.xbuf[1], L, false)) {
             set_error("tensor map of the state frames rejected");
             return cudaErrorInvalidValue;
         }
@@ -430,7 +409,7 @@ cudaError_t conv_tc_prepare(Layer& L)
         set_error("tensor map of the weights rejected (%d)", (int)r);
         return cudaErrorInvalidValue;
     }
-    L.tc_z_tma = encode_z_map(&L.tmap_z, L) ? 1 : 0;
+    L.tc_z_tma = tc_encode_z_map(&L.tmap_z, L) ? 1 : 0;
     const int HH = 8 + L.p.k_h - 1, WW = 8 + L.p.k_w - 1;
     return cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)tc_smem_bytes(HH, WW));
@@ -440,13 +419,13 @@ cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, 
 {
     (void)x_prev;
     alignas(64) CUtensorMap tm_xt;
-    if (!encode_x_map(&tm_xt, x_t, L, L.tc_x5d != 0)) {
+    if (!tc_encode_x_map(&tm_xt, x_t, L, L.tc_x5d != 0)) {
         set_error("tensor map of x_t rejected");
         return cudaErrorInvalidValue;
     }
     TcArgs a;
     a.list = L.list;
-    a.counters = L.counters;
+    a.counters = step_count(L);
     a.z = L.z;
     a.y = (__nv_bfloat16*)L.y;
     a.err = L.err_dev;

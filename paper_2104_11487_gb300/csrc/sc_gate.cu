@@ -1,19 +1,24 @@
-// Gate kernels of the Skip-Conv step.
+// Gate kernels of the Skip-Conv step (two launches).
 //
-// gate_pixel : one pass over x_t and x_{t-1} (the two full-frame reads of the
-//              step).  Per input pixel it forms the residual r_t = x_t - x_{t-1}
-//              (Eq. 2), its l1 norm over all input channels (the channel part of
-//              the Input-Norm gate, Eq. 5, p = 1), and whether the pixel changed
-//              bit-wise.  It also commits x_t into the ping-pong buffer that
-//              becomes x_{t-1} at the next step, writing only pixels that
-//              changed at this step or the previous one (every other pixel of
-//              that buffer already holds x_t).
-// gate_block : one warp per b x b output block.  Per output location it sums
-//              the per-pixel l1 norms over the k_h x k_w receptive field (stride,
-//              zero padding) — the local support norm of Eq. 5 — takes the
-//              block maximum (max-pooling of the gate, Sec. 3.2) and compares it
-//              with the threshold; open blocks are appended to a compact list
-//              with one atomic per CTA.
+// Pass 1, per input pixel: the residual r_t = x_t - x_{t-1} (Eq. 2), its l1
+// norm over all input channels (the channel part of the Input-Norm gate,
+// Eq. 5, p = 1), and whether the pixel changed bit-wise.  The same pass
+// commits x_t into the ping-pong buffer that becomes x_{t-1} at the next step,
+// writing only pixels that changed at this step or the previous one (every
+// other pixel of that buffer already holds x_t).
+//
+// Pass 2, per output block: the per-pixel norms summed over each output
+// location's k_h x k_w receptive field (stride, zero padding) give the local
+// support norm of Eq. 5; the block maximum (max-pooling of the gate,
+// Sec. 3.2 on structured sparsity) is compared with the threshold and open
+// blocks are appended to a compact list with one atomic per eight blocks.
+//
+// Pass 2 is a programmatic dependent launch of pass 1 (its launch latency
+// hides behind pass 1's tail), and the convolution is one of pass 2.
+// A single-launch form was tried: CTAs that publish a band of norms and let
+// the last arriving band evaluate the block row spend about as long on the
+// publication (fence, atomic, barrier) as on the streaming itself at these
+// frame sizes, and were twice as slow.
 #include "sc_internal.h"
 
 namespace sc {
@@ -47,72 +52,104 @@ __device__ __forceinline__ unsigned bits_differ(const uint4& a, const uint4& b)
     return (a.x ^ b.x) | (a.y ^ b.y) | (a.z ^ b.z) | (a.w ^ b.w);
 }
 
-// 16-byte vector path: a pixel's channels are `cpp` 16-byte chunks, handled
-// by a group of G = 2^log2g lanes (each lane up to PER chunks).  Each warp
-// iteration covers U consecutive groups of pixels so that 2*U*PER loads per
-// lane are in flight before the first reduction.
-template <typename T, int PER, int U>
+struct GateGeom {
+    int n, H, W, Ho, Wo, KH, KW, stride, pad, b, nby, nbx;
+};
+
+// Max over the block's output locations of the support sum of per-pixel
+// norms (one warp, returns the same value in every lane).  P is read from L2
+// (other CTAs wrote it during this launch).
+__device__ __forceinline__ float block_score(const GateGeom& g, const float* __restrict__ P, int nn, int by, int bx,
+                                             int lane)
+{
+    const float* Pn = P + (size_t)nn * g.H * g.W;
+    const int bh = min(g.b, g.Ho - by * g.b), bw = min(g.b, g.Wo - bx * g.b);
+    const int fy0 = by * g.b * g.stride - g.pad, fx0 = bx * g.b * g.stride - g.pad;
+    float best = -1.f;
+    for (int q = lane; q < bh * bw; q += 32) {
+        const int i = q / bw, j = q - (q / bw) * bw;
+        float S = 0.f;
+        for (int kh = 0; kh < g.KH; ++kh) {
+            const int yy = fy0 + i * g.stride + kh;
+            if (yy < 0 || yy >= g.H) continue;
+            for (int kw = 0; kw < g.KW; ++kw) {
+                const int xx = fx0 + j * g.stride + kw;
+                if (xx < 0 || xx >= g.W) continue;
+                S += __ldcg(Pn + (size_t)yy * g.W + xx);
+            }
+        }
+        best = fmaxf(best, S);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+    return best;
+}
+
+// Vector path, pass 1 of 2: every warp of a grid-stride grid takes groups of
+// pixels (G lanes per pixel, PER 16-byte chunks per lane); the change flag of
+// the previous step is loaded together with the frames.  The last thing each
+// CTA does is let the block-gate pass start (programmatic dependent launch).
+template <typename T, int PER>
 __global__ void __launch_bounds__(256) gate_pixel_vec_kernel(
     const uint4* __restrict__ xt, const uint4* __restrict__ xp, uint4* __restrict__ xn,
     const uint8_t* __restrict__ chg_prev, uint8_t* __restrict__ chg_cur, float* __restrict__ pix_l1,
-    long long n_pix, int cpp, int log2g, int32_t* __restrict__ counters)
+    long long n_pix, int cpp, int log2g, int32_t* __restrict__ count_cur, int32_t* __restrict__ count_next)
 {
-    if (blockIdx.x == 0 && threadIdx.x == 0) counters[0] = 0;  // reset the active-block count
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        *count_cur = 0;   // this step's active-block count (filled by the block-gate pass)
+        *count_next = 0;
+    }
     const int lane = threadIdx.x & 31;
     const int G = 1 << log2g;
     const int sub = lane & (G - 1);
     const int gpw = 32 >> log2g;
     const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    for (long long base = warp * gpw * U; base < n_pix; base += nwarps * gpw * U) {
-        uint4 a[U][PER], b[U][PER];
+    for (long long base = warp * gpw; base < n_pix; base += nwarps * gpw) {
+        const long long pix = base + (lane >> log2g);
+        const bool valid = pix < n_pix;
+        uint4 a[PER], b[PER];
+        const uint8_t cprev = valid ? __ldg(chg_prev + pix) : (uint8_t)0;
 #pragma unroll
-        for (int v = 0; v < U; ++v) {
-            const long long pix = base + v * gpw + (lane >> log2g);
-#pragma unroll
-            for (int k = 0; k < PER; ++k) {
-                const int c = sub + k * G;
-                if (pix < n_pix && c < cpp) {
-                    a[v][k] = __ldg(xt + pix * cpp + c);
-                    b[v][k] = __ldg(xp + pix * cpp + c);
-                } else {
-                    a[v][k] = make_uint4(0, 0, 0, 0);
-                    b[v][k] = make_uint4(0, 0, 0, 0);
-                }
+        for (int k = 0; k < PER; ++k) {
+            const int c = sub + k * G;
+            if (valid && c < cpp) {
+                a[k] = __ldg(xt + pix * cpp + c);
+                b[k] = __ldg(xp + pix * cpp + c);
+            } else {
+                a[k] = make_uint4(0, 0, 0, 0);
+                b[k] = make_uint4(0, 0, 0, 0);
             }
         }
+        float s = 0.f;
+        unsigned diff = 0;
 #pragma unroll
-        for (int v = 0; v < U; ++v) {
-            const long long pix = base + v * gpw + (lane >> log2g);
-            float s = 0.f;
-            unsigned diff = 0;
+        for (int k = 0; k < PER; ++k) {
+            s += l1_diff(a[k], b[k], (T*)nullptr);
+            diff |= bits_differ(a[k], b[k]);
+        }
 #pragma unroll
-            for (int k = 0; k < PER; ++k) {
-                s += l1_diff(a[v][k], b[v][k], (T*)nullptr);
-                diff |= bits_differ(a[v][k], b[v][k]);
+        for (int off = 16; off > 0; off >>= 1) {
+            if (off < G) {
+                s += __shfl_xor_sync(0xffffffffu, s, off);
+                diff |= __shfl_xor_sync(0xffffffffu, diff, off);
             }
+        }
+        if (valid) {
+            if (diff || cprev) {
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-                if (off < G) {
-                    s += __shfl_xor_sync(0xffffffffu, s, off);
-                    diff |= __shfl_xor_sync(0xffffffffu, diff, off);
+                for (int k = 0; k < PER; ++k) {
+                    const int c = sub + k * G;
+                    if (c < cpp) xn[pix * cpp + c] = a[k];
                 }
             }
-            if (pix < n_pix) {
-                if (diff || chg_prev[pix]) {
-#pragma unroll
-                    for (int k = 0; k < PER; ++k) {
-                        const int c = sub + k * G;
-                        if (c < cpp) xn[pix * cpp + c] = a[v][k];
-                    }
-                }
-                if (sub == 0) {
-                    pix_l1[pix] = s;
-                    chg_cur[pix] = diff ? 1 : 0;
-                }
+            if (sub == 0) {
+                pix_l1[pix] = s;
+                chg_cur[pix] = diff ? 1 : 0;
             }
         }
     }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // Element path for channel counts whose pixel is not a multiple of 16 bytes.
@@ -120,9 +157,12 @@ template <typename T, int PER>
 __global__ void __launch_bounds__(256) gate_pixel_elem_kernel(
     const T* __restrict__ xt, const T* __restrict__ xp, T* __restrict__ xn,
     const uint8_t* __restrict__ chg_prev, uint8_t* __restrict__ chg_cur, float* __restrict__ pix_l1,
-    long long n_pix, int C, int log2g, int32_t* __restrict__ counters)
+    long long n_pix, int C, int log2g, int32_t* __restrict__ count_cur, int32_t* __restrict__ count_next)
 {
-    if (blockIdx.x == 0 && threadIdx.x == 0) counters[0] = 0;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        *count_cur = 0;
+        *count_next = 0;
+    }
     const int lane = threadIdx.x & 31;
     const int G = 1 << log2g;
     const int sub = lane & (G - 1);
@@ -171,63 +211,61 @@ __global__ void __launch_bounds__(256) gate_pixel_elem_kernel(
             }
         }
     }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// One warp per gate block.  The block's input footprint of per-pixel norms
-// (FH x FW with FH = (b-1)*stride + k_h) is staged in shared memory with one
-// round of coalesced loads; each lane then box-sums the supports of its
-// output locations from shared memory.  When the footprint is too large for
-// the staging area (stage == 0) the sums read global memory directly.
-__global__ void __launch_bounds__(256) gate_block_kernel(
-    const float* __restrict__ pix_l1, uint8_t* __restrict__ mask, int32_t* __restrict__ list,
-    int32_t* __restrict__ counters, int n, int H, int W, int Ho, int Wo, int KH, int KW, int stride, int pad,
-    int b, int nby, int nbx, float thr, int force, int stage)
+// One warp per gate block (two-launch form).
+// Pass 2: one warp per gate block.  Launched as a programmatic dependent of
+// pass 1: it waits for pass 1's results before reading them, and lets the
+// convolution after it start its own prologue right away.  When the block's
+// footprint of norms fits (stage), it is staged in shared memory with one
+// round of loads.
+__global__ void __launch_bounds__(256) gate_block_kernel(const float* __restrict__ pix_l1, uint8_t* __restrict__ mask,
+                                                         int32_t* __restrict__ list, int32_t* __restrict__ count_cur,
+                                                         GateGeom g, float thr, int force, int stage)
 {
-    extern __shared__ float foot[];  // [8 warps][FH*FW] when staging
+    extern __shared__ float foot[];  // [8 warps][FH * FW]
     __shared__ int flags[8];
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const long long nblocks = (long long)n * nby * nbx;
+    const long long nblocks = (long long)g.n * g.nby * g.nbx;
     const long long blk = (long long)blockIdx.x * 8 + wid;
-    const int FH = (b - 1) * stride + KH, FW = (b - 1) * stride + KW;
     int open = 0;
     if (blk < nblocks) {
         if (force) {
             open = 1;
         } else {
-            const int bx = (int)(blk % nbx);
-            const long long rest = blk / nbx;
-            const int by = (int)(rest % nby);
-            const int nn = (int)(rest / nby);
-            const float* P = pix_l1 + (size_t)nn * H * W;
-            const int bh = min(b, Ho - by * b), bw = min(b, Wo - bx * b);
-            const int fy0 = by * b * stride - pad, fx0 = bx * b * stride - pad;
-            float* F = foot + wid * FH * FW;
+            const int bx = (int)(blk % g.nbx);
+            const long long rest = blk / g.nbx;
+            const int by = (int)(rest % g.nby);
+            const int nn = (int)(rest / g.nby);
             if (stage) {
+                // block footprint (FH x FW) into this warp's slice of shared memory
+                const int FH = (g.b - 1) * g.stride + g.KH, FW = (g.b - 1) * g.stride + g.KW;
+                float* F = foot + wid * FH * FW;
+                const float* Pn = pix_l1 + (size_t)nn * g.H * g.W;
+                const int fy0 = by * g.b * g.stride - g.pad, fx0 = bx * g.b * g.stride - g.pad;
                 for (int q = lane; q < FH * FW; q += 32) {
                     const int yy = fy0 + q / FW, xx = fx0 + q % FW;
-                    F[q] = (yy >= 0 && yy < H && xx >= 0 && xx < W) ? __ldg(P + (size_t)yy * W + xx) : 0.f;
+                    F[q] = (yy >= 0 && yy < g.H && xx >= 0 && xx < g.W) ? __ldcg(Pn + (size_t)yy * g.W + xx) : 0.f;
                 }
                 __syncwarp();
-            }
-            float best = -1.f;
-            for (int q = lane; q < bh * bw; q += 32) {
-                const int i = q / bw, j = q % bw;  // within the block
-                float S = 0.f;
-                for (int kh = 0; kh < KH; ++kh)
-                    for (int kw = 0; kw < KW; ++kw) {
-                        const int fy = i * stride + kh, fx = j * stride + kw;
-                        if (stage) {
-                            S += F[fy * FW + fx];
-                        } else {
-                            const int yy = fy0 + fy, xx = fx0 + fx;
-                            if (yy >= 0 && yy < H && xx >= 0 && xx < W) S += __ldg(P + (size_t)yy * W + xx);
-                        }
-                    }
-                best = fmaxf(best, S);
-            }
+                const int bh = min(g.b, g.Ho - by * g.b), bw = min(g.b, g.Wo - bx * g.b);
+                float best = -1.f;
+                for (int q = lane; q < bh * bw; q += 32) {
+                    const int i = q / bw, j = q - (q / bw) * bw;
+                    float S = 0.f;
+                    for (int kh = 0; kh < g.KH; ++kh)
+                        for (int kw = 0; kw < g.KW; ++kw) S += F[(i * g.stride + kh) * FW + j * g.stride + kw];
+                    best = fmaxf(best, S);
+                }
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
-            open = best > thr ? 1 : 0;
+                for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+                open = best > thr ? 1 : 0;
+            } else {
+                open = block_score(g, pix_l1, nn, by, bx, lane) > thr ? 1 : 0;
+            }
         }
         if (lane == 0) mask[blk] = (uint8_t)open;
     }
@@ -237,17 +275,36 @@ __global__ void __launch_bounds__(256) gate_block_kernel(
         const int f = lane < 8 ? flags[lane] : 0;
         const unsigned bal = __ballot_sync(0xffffffffu, f);
         int base = 0;
-        if (lane == 0 && bal) base = atomicAdd(&counters[0], __popc(bal));
+        if (lane == 0 && bal) base = atomicAdd(count_cur, __popc(bal));
         base = __shfl_sync(0xffffffffu, base, 0);
         if (f) list[base + __popc(bal & ((1u << lane) - 1u))] = (int32_t)(blockIdx.x * 8 + lane);
     }
 }
 
-template <typename T>
-cudaError_t launch_pixel_typed(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
-                               const uint8_t* chg_prev, uint8_t* chg_cur)
+GateGeom geom_of(const Layer& L)
 {
-    const long long n_pix = (long long)L.p.n_streams * L.p.h * L.p.w;
+    GateGeom g;
+    g.n = L.p.n_streams;
+    g.H = L.p.h;
+    g.W = L.p.w;
+    g.Ho = L.ho;
+    g.Wo = L.wo;
+    g.KH = L.p.k_h;
+    g.KW = L.p.k_w;
+    g.stride = L.p.stride;
+    g.pad = L.p.pad;
+    g.b = L.p.block;
+    g.nby = L.nby;
+    g.nbx = L.nbx;
+    return g;
+}
+
+template <typename T>
+cudaError_t launch_typed(const Layer& L, const void* x_t, const void* x_prev, void* x_next, const uint8_t* chg_prev,
+                         uint8_t* chg_cur, int force)
+{
+    int32_t* cnt_cur = step_count(L);
+    int32_t* cnt_next = next_count(L);
     const int bytes = L.p.c_in * (int)sizeof(T);
     const bool vec = (bytes % 16 == 0) && ((uintptr_t)x_t % 16 == 0) && ((uintptr_t)x_prev % 16 == 0) &&
                      ((uintptr_t)x_next % 16 == 0);
@@ -256,41 +313,58 @@ cudaError_t launch_pixel_typed(const Layer& L, const void* x_t, const void* x_pr
     while ((1 << log2g) < units && log2g < 5) ++log2g;
     const int G = 1 << log2g;
     const int per = (units + G - 1) / G;
+    const GateGeom g = geom_of(L);
+    const long long n_pix = (long long)L.p.n_streams * L.p.h * L.p.w;
     const int gpw = 32 / G;
-    long long warps_needed = (n_pix + gpw - 1) / gpw;
-    long long blocks = (warps_needed + 7) / 8;
+    const long long warps_needed = (n_pix + gpw - 1) / gpw;
+    const long long blocks = (warps_needed + 7) / 8;
     const long long cap = (long long)L.num_sms * 8;
     const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
     if (vec) {
         const uint4* a = (const uint4*)x_t;
         const uint4* b = (const uint4*)x_prev;
         uint4* c = (uint4*)x_next;
-        if (per == 1)
-            gate_pixel_vec_kernel<T, 1, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per == 2)
-            gate_pixel_vec_kernel<T, 2, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per <= 4)
-            gate_pixel_vec_kernel<T, 4, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else
-            return cudaErrorInvalidValue;
+#define SC_VEC(PER_)                                                                                             \
+    gate_pixel_vec_kernel<T, PER_><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, \
+                                                               log2g, cnt_cur, cnt_next)
+        if (per == 1) SC_VEC(1);
+        else if (per == 2) SC_VEC(2);
+        else if (per <= 4) SC_VEC(4);
+        else return cudaErrorInvalidValue;
+#undef SC_VEC
     } else {
-        const T* a = (const T*)x_t;
-        const T* b = (const T*)x_prev;
-        T* c = (T*)x_next;
-        if (per == 1)
-            gate_pixel_elem_kernel<T, 1><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per == 2)
-            gate_pixel_elem_kernel<T, 2><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per <= 4)
-            gate_pixel_elem_kernel<T, 4><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per <= 8)
-            gate_pixel_elem_kernel<T, 8><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else if (per <= 32)
-            gate_pixel_elem_kernel<T, 32><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, log2g, L.counters);
-        else
-            return cudaErrorInvalidValue;
+    const T* a = (const T*)x_t;
+    const T* b = (const T*)x_prev;
+    T* c = (T*)x_next;
+#define SC_ELEM(PER_)                                                                                              \
+    gate_pixel_elem_kernel<T, PER_><<<grid, 256, 0, L.stream>>>(a, b, c, chg_prev, chg_cur, L.pix_l1, n_pix, units, \
+                                                                log2g, cnt_cur, cnt_next)
+    if (per == 1) SC_ELEM(1);
+    else if (per == 2) SC_ELEM(2);
+    else if (per <= 4) SC_ELEM(4);
+    else if (per <= 8) SC_ELEM(8);
+    else if (per <= 32) SC_ELEM(32);
+    else return cudaErrorInvalidValue;
+#undef SC_ELEM
     }
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const long long nblocks = (long long)L.p.n_streams * L.nby * L.nbx;
+    const int FH = (L.p.block - 1) * L.p.stride + L.p.k_h, FW = (L.p.block - 1) * L.p.stride + L.p.k_w;
+    const size_t foot = (size_t)8 * FH * FW * sizeof(float);
+    const int stage = foot <= 40 * 1024 ? 1 : 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((nblocks + 7) / 8));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = stage ? foot : 0;
+    cfg.stream = L.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gate_block_kernel, (const float*)L.pix_l1, L.mask, L.list, cnt_cur, g,
+                              L.gate_thr, force, stage);
 }
 
 }  // namespace
@@ -303,25 +377,12 @@ int gate_max_channels(int dtype, bool vec)
     return vec ? (32 * 4 * 16) / es : 32 * 32;
 }
 
-cudaError_t launch_gate_pixel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
-                              const uint8_t* chg_prev, uint8_t* chg_cur)
+cudaError_t launch_gate(const Layer& L, const void* x_t, const void* x_prev, void* x_next, const uint8_t* chg_prev,
+                        uint8_t* chg_cur, int force)
 {
     if (L.p.dtype == SKIPCONV_BF16)
-        return launch_pixel_typed<__nv_bfloat16>(L, x_t, x_prev, x_next, chg_prev, chg_cur);
-    return launch_pixel_typed<float>(L, x_t, x_prev, x_next, chg_prev, chg_cur);
-}
-
-cudaError_t launch_gate_block(const Layer& L, int force)
-{
-    const long long nblocks = (long long)L.p.n_streams * L.nby * L.nbx;
-    const int grid = (int)((nblocks + 7) / 8);
-    const int FH = (L.p.block - 1) * L.p.stride + L.p.k_h, FW = (L.p.block - 1) * L.p.stride + L.p.k_w;
-    const size_t foot = (size_t)8 * FH * FW * sizeof(float);
-    const int stage = foot <= 40 * 1024 ? 1 : 0;
-    gate_block_kernel<<<grid, 256, stage ? foot : 0, L.stream>>>(
-        L.pix_l1, L.mask, L.list, L.counters, L.p.n_streams, L.p.h, L.p.w, L.ho, L.wo, L.p.k_h, L.p.k_w,
-        L.p.stride, L.p.pad, L.p.block, L.nby, L.nbx, L.gate_thr, force, stage);
-    return cudaGetLastError();
+        return launch_typed<__nv_bfloat16>(L, x_t, x_prev, x_next, chg_prev, chg_cur, force);
+    return launch_typed<float>(L, x_t, x_prev, x_next, chg_prev, chg_cur, force);
 }
 
 }  // namespace sc

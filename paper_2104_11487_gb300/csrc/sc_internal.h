@@ -31,7 +31,7 @@ struct Layer {
     float* pix_l1;          // per input pixel: sum over channels of |r| (scratch)
     uint8_t* mask;          // [n][nby][nbx]
     int32_t* list;          // active block ids
-    int32_t* counters;      // [0] active count, [1..] scratch counters
+    int32_t* counters;      // [0], [1]: active-block count of even / odd steps
     float* z;               // [n][ho][wo][c_out]
     void* y;                // [n][ho][wo][c_out] dtype or NULL
     float* bias;            // [c_out]
@@ -61,15 +61,21 @@ struct Layer {
     int tc_x5d;             // 1: halo tiles as one 5-D TMA box per channel chunk; 0: 4-D boxes per 8 channels
     CUtensorMap tmap_xbuf[2];
     CUtensorMap tmap_w;
+    int tc_ws;              // 1: use the weight-stationary kernel
+    CUtensorMap tmap_xrow[2];  // weight-stationary kernel: 128-byte-row halo boxes of the state frames
     int tc_z_tma;           // 1: the z tensor map below is valid (c_out multiple of 4)
     CUtensorMap tmap_z;
 };
 
 // ------------------------------------------------------------------ launchers
-// Gate (sc_gate.cu)
-cudaError_t launch_gate_pixel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
-                              const uint8_t* chg_prev, uint8_t* chg_cur);
-cudaError_t launch_gate_block(const Layer& L, int force);
+// Active-block count of the step being enqueued (step t uses slot t % 2; the
+// gate of step t clears slot (t+1) % 2 for the next step).
+inline int32_t* step_count(const Layer& L) { return L.counters + (L.t & 1); }
+inline int32_t* next_count(const Layer& L) { return L.counters + ((L.t + 1) & 1); }
+
+// Gate (sc_gate.cu): residual norms, state commit, block gates and the open-block list
+cudaError_t launch_gate(const Layer& L, const void* x_t, const void* x_prev, void* x_next, const uint8_t* chg_prev,
+                        uint8_t* chg_cur, int force);
 
 // CUDA-core convolution and elementwise kernels (sc_conv_cc.cu)
 cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
@@ -82,6 +88,11 @@ size_t conv_cc_smem_bytes(const Layer& L);
 bool conv_tc_supported(const skipconv_params& p, const char** why);
 cudaError_t conv_tc_prepare(Layer& L);     // tensor maps of the state buffers and weights
 cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, int prev_index);
+
+// Weight-stationary tensor-core convolution (sc_conv_ws.cu), for layers that keep no y
+bool conv_ws_supported(const Layer& L);
+cudaError_t conv_ws_prepare(Layer& L);
+cudaError_t launch_conv_ws(const Layer& L, const void* x_t, int prev_index);
 
 // Driver entry point for tensor-map encoding (resolved once through the runtime).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

@@ -1,0 +1,45 @@
+// Pieces shared by the two tensor-core convolution kernels.
+#pragma once
+
+#include "sc_internal.h"
+
+namespace sc {
+
+constexpr int TC_M = 128;   // output channels per MMA tile
+constexpr int TC_N = 64;    // output pixels per MMA tile: one 8x8 gate block
+constexpr int TC_CK = 64;   // input channels per K chunk
+constexpr int TC_ZBYTES = TC_N * TC_M * 4;  // fp32 staging tile of one unit's result
+
+// Bytes of one halo tile (one tensor, one 64-channel chunk) in the no-swizzle
+// K-major canonical layout [8-channel group][row][col][8 channels].
+__host__ __device__ inline int x_tile_bytes(int HH, int WW) { return 8 * HH * WW * 16; }
+
+// Open-block id -> (stream, block row, block column).
+__device__ __forceinline__ void decode_block(int id, int nby, int nbx, int& n, int& by, int& bx)
+{
+    bx = id % nbx;
+    by = (id / nbx) % nby;
+    n = id / (nbx * nby);
+}
+
+// Eight bf16 residuals x - p, formed in fp32 and rounded to nearest.
+__device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
+{
+    const __nv_bfloat162* a = reinterpret_cast<const __nv_bfloat162*>(&x);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&p);
+    uint4 out;
+    __nv_bfloat162* o = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 fa = __bfloat1622float2(a[k]);
+        const float2 fb = __bfloat1622float2(b[k]);
+        o[k] = __floats2bfloat162_rn(fa.x - fb.x, fa.y - fb.y);
+    }
+    return out;
+}
+
+// Tensor maps (sc_conv_tc.cu): halo boxes of a frame, and the z state.
+bool tc_encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d);
+bool tc_encode_z_map(CUtensorMap* m, const Layer& L);
+
+}  // namespace sc

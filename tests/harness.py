@@ -91,12 +91,12 @@ def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_
 
 
 def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
-                     reset_at=()):
+                     reset_at=(), emit_y=False):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record."""
     import oracle
     ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode)
-    gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path)
+    gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y)
     cmp = Compare(spec, dtype, name)
     try:
         for t, f in enumerate(frames):
@@ -110,6 +110,12 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
             mask, lst, cnt = gl.gate()
             cmp.frame(t, score, mask_ref, mask.cpu().numpy(), lst.cpu().numpy(), cnt, ref.z,
                       gl.z().cpu().numpy().astype(np.float64), forced)
+            if emit_y:
+                y_gpu = gl.y().float().cpu().numpy().astype(np.float64)
+                y_ref = oracle.layer_output(ref.z, None, 0, 2 if dtype == "bf16" else 1)
+                rms = float(np.sqrt(np.mean(y_ref ** 2)))
+                allowed = (TOL_BF16_REL_RMS * rms if dtype == "bf16" else TOL_F32_ABS) + np.abs(y_ref) * 2.0 ** -7
+                assert (np.abs(y_gpu - y_ref) <= allowed).all(), "%s t=%d: y beyond tolerance" % (name, t)
             if check_prev:
                 import torch
                 assert torch.equal(gl.prev_input().view(torch.int16 if dtype == "bf16" else torch.int32),

@@ -44,6 +44,15 @@ def test_c1_bf16_8x8_blocks(path):
     assert cmp.frames == 16
 
 
+def test_c1_streaming_tensor_core_kernel_with_y():
+    """A layer that keeps y = act(z) runs the streaming tensor-core kernel
+    (the weight-stationary one adds partial sums into z and keeps no y)."""
+    wl = synth.make_workload("c1")
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                                 emit_y=True, name="c1+y")
+    assert used == TENSOR_CORE and cmp.frames == 16
+
+
 def test_c2_pose_stack_teacher_forced():
     wl = synth.make_workload("c2")
     cmps, paths = run_stack_teacher_forced(wl)
