@@ -368,10 +368,15 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     const int cur = (int)(L->t & 1), nxt = cur ^ 1;
     // xbuf[cur] holds x_{t-1}; xbuf[nxt] holds x_{t-2} and receives x_t.
     // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
+    const int force = (L->key || L->p.dense_mode) ? 1 : 0;
     int slot = prof_begin(L, 0);
-    cudaError_t e = launch_gate(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur],
-                                (L->key || L->p.dense_mode) ? 1 : 0);
+    cudaError_t e = launch_gate_pixels(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur], force);
     prof_end(L, slot);
+    if (e == cudaSuccess) {
+        slot = prof_begin(L, 1);
+        e = launch_gate_blocks(*L, force);
+        prof_end(L, slot);
+    }
     if (e == cudaSuccess) {
         slot = prof_begin(L, 2);
         if (L->path == SKIPCONV_PATH_TENSOR_CORE && L->tc_ws) e = launch_conv_ws(*L, x_t, cur);

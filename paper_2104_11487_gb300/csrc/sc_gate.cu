@@ -347,8 +347,16 @@ cudaError_t launch_typed(const Layer& L, const void* x_t, const void* x_prev, vo
     else return cudaErrorInvalidValue;
 #undef SC_ELEM
     }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    (void)force;
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gate_blocks(const Layer& L, int force)
+{
+    int32_t* cnt_cur = step_count(L);
+    const GateGeom g = geom_of(L);
     const long long nblocks = (long long)L.p.n_streams * L.nby * L.nbx;
     const int FH = (L.p.block - 1) * L.p.stride + L.p.k_h, FW = (L.p.block - 1) * L.p.stride + L.p.k_w;
     const size_t foot = (size_t)8 * FH * FW * sizeof(float);
@@ -367,8 +375,6 @@ cudaError_t launch_typed(const Layer& L, const void* x_t, const void* x_prev, vo
                               L.gate_thr, force, stage);
 }
 
-}  // namespace
-
 // Largest channel count the gate kernels take (per pixel: 4 chunks of 16 B
 // per lane on the vector path, 32 elements per lane on the element path).
 int gate_max_channels(int dtype, bool vec)
@@ -377,8 +383,8 @@ int gate_max_channels(int dtype, bool vec)
     return vec ? (32 * 4 * 16) / es : 32 * 32;
 }
 
-cudaError_t launch_gate(const Layer& L, const void* x_t, const void* x_prev, void* x_next, const uint8_t* chg_prev,
-                        uint8_t* chg_cur, int force)
+cudaError_t launch_gate_pixels(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
+                               const uint8_t* chg_prev, uint8_t* chg_cur, int force)
 {
     if (L.p.dtype == SKIPCONV_BF16)
         return launch_typed<__nv_bfloat16>(L, x_t, x_prev, x_next, chg_prev, chg_cur, force);

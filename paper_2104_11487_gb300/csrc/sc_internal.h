@@ -73,9 +73,11 @@ struct Layer {
 inline int32_t* step_count(const Layer& L) { return L.counters + (L.t & 1); }
 inline int32_t* next_count(const Layer& L) { return L.counters + ((L.t + 1) & 1); }
 
-// Gate (sc_gate.cu): residual norms, state commit, block gates and the open-block list
-cudaError_t launch_gate(const Layer& L, const void* x_t, const void* x_prev, void* x_next, const uint8_t* chg_prev,
-                        uint8_t* chg_cur, int force);
+// Gate (sc_gate.cu): pass 1, residual norms per pixel and the state commit;
+// pass 2, block gates and the open-block list (a programmatic dependent of pass 1)
+cudaError_t launch_gate_pixels(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
+                               const uint8_t* chg_prev, uint8_t* chg_cur, int force);
+cudaError_t launch_gate_blocks(const Layer& L, int force);
 
 // CUDA-core convolution and elementwise kernels (sc_conv_cc.cu)
 cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
