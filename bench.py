@@ -190,19 +190,33 @@ def make_layer(wl, torch, dense_mode=False):
                          dense_mode=dense_mode, weights=torch.from_numpy(wl.weights[0]), bias=None)
 
 
+PROFILE_FILES = {"gate_pixel": ("gate_pixel", "sc_gate.cu"), "gate_block": ("gate_block", "sc_gate.cu"),
+                 "conv": ("conv_ws", "sc_conv_ws.cu")}
+
+
 def traffic_from_profiles(kernel):
-    """dram bytes per launch from the committed ncu summary of `kernel` on
-    this workload, when one exists for the current kernel source."""
-    path = os.path.join(ROOT, "profiles", "%s_c4_d10.md" % kernel)
+    """DRAM bytes per launch of `kernel` from its committed ncu summary on
+    this workload, or None when there is none or the kernel's source has
+    changed since the counters were taken (the summary records the sha256 of
+    the source file it was captured from)."""
+    import hashlib
+    if kernel not in PROFILE_FILES:
+        return None
+    name, src = PROFILE_FILES[kernel]
+    path = os.path.join(ROOT, "profiles", "%s_c4_d10.md" % name)
     if not os.path.exists(path):
         return None
+    digest = hashlib.sha256(open(os.path.join(ROOT, "paper_2104_11487_gb300", "csrc", src), "rb").read()).hexdigest()
+    traffic, source_ok = None, False
     for line in open(path):
         if line.startswith("dram_bytes_per_launch:"):
             try:
-                return float(line.split(":", 1)[1].split()[0])
+                traffic = float(line.split(":", 1)[1].split()[0])
             except ValueError:
-                return None
-    return None
+                traffic = None
+        if line.startswith("source_sha256:") and line.split(":", 1)[1].strip().split()[0] == digest:
+            source_ok = True
+    return traffic if source_ok else None
 
 
 # ----------------------------------------------------------- CPU oracle
