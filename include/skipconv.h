@@ -174,6 +174,45 @@ SKIPCONV_API int skipconv_profile(skipconv_handle h, int enable);
  * (milliseconds are 0 unless timing was enabled). */
 SKIPCONV_API int skipconv_profile_read(skipconv_handle h, long long* launches, double* ms);
 
+/* Largest n_streams*h*w that skipconv_gate_noalloc accepts: its static device
+ * scratch holds one float32 norm per input pixel (4 MiB + 256 B per device). */
+#define SKIPCONV_NOALLOC_MAX_PIXELS (1 << 20)
+
+/* Block gate of one frame pair, with no allocation of any kind.  The paper has
+ * no counterpart: this is a deployment form of the gate that skipconv_step
+ * runs, for callers that must not allocate device memory while they run -- a
+ * process whose device memory is held by a caching allocator (cudaMalloc may
+ * fail there, or force the cache to shrink) and latency-bound callers that
+ * cannot take the device-wide synchronisation of cudaMalloc/cudaFree.  It
+ * needs no handle.  It computes, for r = x_t - x_prev (Eq. 2), the l1 norm of
+ * r over each output location's c_in x k_h x k_w support (Eq. 5, stride and
+ * zero padding as in params), its maximum over each b x b block (Sec. 3.2),
+ * and opens the blocks above the threshold of params->gate (INPUT_MEAN or
+ * INPUT_SUM; dense_mode = 1 opens every block).  The convolution fields of
+ * params are validated as for skipconv_create and otherwise unused.
+ *   x_t, x_prev  : device frames [n][h][w][c_in] in dtype (read only)
+ *   block_mask   : device uint8 [n][nby][nbx], written
+ *   active_list  : device int32 with room for n*nby*nbx ids; the open block
+ *                  ids, order unspecified
+ *   active_count : device int32, the number of open blocks
+ *   stream       : cudaStream_t (NULL = legacy default stream)
+ * Enqueued on `stream`; returns without waiting.  Scratch: one static
+ * __device__ array of 256 + 4*SKIPCONV_NOALLOC_MAX_PIXELS bytes per device.
+ * The first call on a device (with that device current) performs the set-up:
+ * it takes the array's address with cudaGetSymbolAddress, where the runtime
+ * loads the library's module on that device, and caches it; make that first
+ * call before any stream capture.  Later calls only launch kernels and one
+ * 4-byte device-to-device copy.  The open-block counter in the scratch is
+ * zeroed on the device by every call.  Every call on a device shares the one
+ * scratch: calls whose work may overlap on the device (different streams or
+ * host threads) race and must be serialised by the caller.
+ * Errors: INVALID (NULL pointer, bad params, n_streams*h*w above
+ * SKIPCONV_NOALLOC_MAX_PIXELS), UNSUPPORTED (gate OUTPUT, which needs ||w||_1
+ * that only a handle holds), CUDA (set-up or launch failed). */
+SKIPCONV_API int skipconv_gate_noalloc(const skipconv_params* params, const void* x_t, const void* x_prev,
+                                       uint8_t* block_mask, int32_t* active_list, int32_t* active_count,
+                                       void* stream);
+
 /* Human-readable name of a status code (static string). */
 SKIPCONV_API const char* skipconv_status_string(int status);
 

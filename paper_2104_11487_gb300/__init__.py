@@ -6,6 +6,7 @@ binding whose library cannot be built or loaded raises.
 """
 from ._build import build_library  # noqa: F401
 from .skipconv import (SkipConvLayer, device_tensor, skipconv_check_device, skipconv_create,  # noqa: F401
-                       skipconv_destroy, skipconv_get_gate, skipconv_get_info, skipconv_get_prev_input,
+                       skipconv_destroy, skipconv_gate_noalloc, skipconv_get_gate, skipconv_get_info,
+                       skipconv_get_prev_input,
                        skipconv_get_stats, skipconv_get_y, skipconv_get_z, skipconv_profile, skipconv_profile_read,
                        skipconv_reset_state, skipconv_step, skipconv_step_host)

@@ -37,6 +37,7 @@ SIGNATURES = {
     "skipconv_check_device": (c_int, [c_void_p]),
     "skipconv_profile": (c_int, [c_void_p, c_int]),
     "skipconv_profile_read": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "skipconv_gate_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "skipconv_status_string": (ctypes.c_char_p, [c_int]),
     "skipconv_last_error": (ctypes.c_char_p, []),
 }

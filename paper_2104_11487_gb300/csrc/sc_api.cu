@@ -141,7 +141,7 @@ static int check_device_word(const Layer* L)
     return v == DEV_TIMEOUT ? SKIPCONV_ERR_TIMEOUT : SKIPCONV_ERR_DEVICE;
 }
 
-static int validate(const skipconv_params* p)
+int validate(const skipconv_params* p)
 {
     if (!p) return set_error("params is NULL"), SKIPCONV_ERR_INVALID;
     if (p->n_streams < 1 || p->c_in < 1 || p->c_out < 1 || p->h < 1 || p->w < 1 || p->k_h < 1 || p->k_w < 1 ||

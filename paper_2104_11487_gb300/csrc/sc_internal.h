@@ -103,6 +103,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 EncodeTiledFn encode_tiled_fn();
 
 void set_error(const char* fmt, ...);
+// Host-side check of a parameter block (sizes, enums, limits); sets the error text.
+int validate(const skipconv_params* p);
 
 }  // namespace sc
 

@@ -72,6 +72,12 @@ def skipconv_get_gate(handle: int):
     return m.value, l.value, c.value
 
 
+def skipconv_gate_noalloc(params: Params, x_t, x_prev, block_mask, active_list, active_count, stream=None) -> None:
+    check("skipconv_gate_noalloc", _lib.lib().skipconv_gate_noalloc(
+        ctypes.byref(params), _ptr(x_t), _ptr(x_prev), _ptr(block_mask), _ptr(active_list), _ptr(active_count),
+        _ptr(stream) if stream is not None and not isinstance(stream, int) else stream))
+
+
 def skipconv_get_info(handle: int) -> Info:
     info = Info()
     check("skipconv_get_info", _lib.lib().skipconv_get_info(handle, ctypes.byref(info)))
