@@ -34,7 +34,7 @@ METRIC = "Skip-Conv frames/s and effective TFLOP/s vs roofline at measured gate 
 UNIT = "stream-frames/s"
 N_STREAMS, H, W, C, K, BLOCK, EPS = 8, 128, 128, 256, 3, 8, 0.05
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KERNELS = ("gate_pixel", "gate_block", "conv", "y_refresh")
+KERNELS = ("gate_pixel", "gate_block", "conv", "y_refresh", "step_fused")
 
 
 def parse():
@@ -190,23 +190,31 @@ def make_layer(wl, torch, dense_mode=False):
                          dense_mode=dense_mode, weights=torch.from_numpy(wl.weights[0]), bias=None)
 
 
-PROFILE_FILES = {"gate_pixel": ("gate_pixel", "sc_gate.cu"), "gate_block": ("gate_block", "sc_gate.cu"),
-                 "conv": ("conv_ws", "sc_conv_ws.cu")}
+PROFILE_FILES = {"gate_pixel": ("gate_pixel", ("sc_gate.cu",)), "gate_block": ("gate_block", ("sc_gate.cu",)),
+                 "conv": ("conv_ws", ("sc_conv_ws.cu", "sc_ws_roles.cuh")),
+                 "step_fused": ("step_fused", ("sc_step_fused.cu", "sc_ws_roles.cuh"))}
+
+
+def source_digest(files):
+    import hashlib
+    h = hashlib.sha256()
+    for f in files:
+        h.update(open(os.path.join(ROOT, "paper_2104_11487_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
 
 
 def traffic_from_profiles(kernel):
     """DRAM bytes per launch of `kernel` from its committed ncu summary on
-    this workload, or None when there is none or the kernel's source has
+    this workload, or None when there is none or the kernel's sources have
     changed since the counters were taken (the summary records the sha256 of
-    the source file it was captured from)."""
-    import hashlib
+    the source files it was captured from)."""
     if kernel not in PROFILE_FILES:
         return None
-    name, src = PROFILE_FILES[kernel]
+    name, srcs = PROFILE_FILES[kernel]
     path = os.path.join(ROOT, "profiles", "%s_c4_d10.md" % name)
     if not os.path.exists(path):
         return None
-    digest = hashlib.sha256(open(os.path.join(ROOT, "paper_2104_11487_gb300", "csrc", src), "rb").read()).hexdigest()
+    digest = source_digest(srcs)
     traffic, source_ok = None, False
     for line in open(path):
         if line.startswith("dram_bytes_per_launch:"):
@@ -310,10 +318,23 @@ def main():
     t_step = ms_per_step / 1e3
     t_roof = max(flops / (tc_peak * 1e12), b_alg / (hbm * 1e9))
     per_kernel = {KERNELS[k]: {"launches": launches_p[k], "avg_us": (kms[k] / launches_p[k] * 1e3)
-                               if launches_p[k] else None} for k in range(4)}
-    dom = max(range(3), key=lambda k: kms[k])
+                               if launches_p[k] else None} for k in range(len(KERNELS))}
+    dom = max((0, 1, 2, 4), key=lambda k: kms[k])
     dom_us = kms[dom] / max(1, launches_p[dom]) * 1e3
-    if dom == 2:
+    if dom == 4:
+        # the fused kernel is the whole step: its algorithmic bytes are the step's
+        bound_tc = flops / (tc_peak * 1e12) > b_alg / (hbm * 1e9)
+        if bound_tc:
+            ach = flops / (dom_us * 1e-6) / 1e12
+            roof = {"kernel": "step_fused", "bound": "tensor", "achieved": ach, "peak": tc_peak, "unit": "TFLOP/s",
+                    "frac": ach / tc_peak, "peak_source": pk_src + " bf16_tflops (burst)",
+                    "traffic": traffic_from_profiles("step_fused")}
+        else:
+            ach = b_alg / (dom_us * 1e-6) / 1e9
+            roof = {"kernel": "step_fused", "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                    "frac": ach / hbm, "peak_source": pk_src + " hbm_gbs", "algorithmic_bytes_per_launch": b_alg,
+                    "traffic": traffic_from_profiles("step_fused")}
+    elif dom == 2:
         ach = flops / (dom_us * 1e-6) / 1e12
         roof = {"kernel": "conv", "bound": "tensor", "achieved": ach, "peak": tc_peak, "unit": "TFLOP/s",
                 "frac": ach / tc_peak, "peak_source": pk_src + " bf16_tflops (burst)",
@@ -329,6 +350,7 @@ def main():
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded block-perturbation video)",
             "config": workload_config(args.density),
             "conv_path": {1: "cuda-core", 2: "tensor-core"}.get(info.conv_path),
+            "step_launches": "one fused launch" if info.fused else "separate gate and convolution launches",
             "active_blocks_per_step": active, "block_density_measured": active / (N_STREAMS * (H // BLOCK) ** 2),
             "changed_pixels_per_step": chg,
             "eff_tflops": flops / t_step / 1e12,

@@ -77,7 +77,9 @@ typedef enum { SKIPCONV_ACT_NONE = 0, SKIPCONV_ACT_RELU = 1, SKIPCONV_ACT_SILU =
 typedef enum {
     SKIPCONV_PATH_AUTO = 0,        /* tensor cores where supported, else CUDA cores */
     SKIPCONV_PATH_CUDA_CORE = 1,   /* float32 FMA direct convolution              */
-    SKIPCONV_PATH_TENSOR_CORE = 2  /* tcgen05 implicit GEMM (bf16 in, fp32 accum)  */
+    SKIPCONV_PATH_TENSOR_CORE = 2, /* tcgen05 implicit GEMM (bf16 in, fp32 accum)  */
+    SKIPCONV_PATH_TENSOR_CORE_SEPARATE = 3 /* the same convolution, but never fused with
+                                      the gate: three launches per step           */
 } skipconv_path;
 
 typedef struct {
@@ -149,6 +151,8 @@ typedef struct {
     int conv_path;     /* path actually used: SKIPCONV_PATH_CUDA_CORE or _TENSOR_CORE */
     int num_sms;       /* SMs of the device the handle lives on               */
     size_t state_bytes;/* device bytes held by the handle                     */
+    int fused;         /* 1: each step is one fused launch (gate and convolution
+                          pipelined over the streams), 0: separate launches  */
 } skipconv_info;
 SKIPCONV_API int skipconv_get_info(skipconv_handle h, skipconv_info* info);
 
@@ -165,13 +169,16 @@ SKIPCONV_API int skipconv_check_device(skipconv_handle h);
 
 /* Per-kernel timing.  Kernel kinds: 0 gate_pixel (residual, channel l1 norm,
  * state commit), 1 gate_block (support norm, block gate, compaction), 2 the
- * convolution of the open blocks (either path), 3 y refresh.  Launch counts
- * are always kept; with enable = 1 each launch is also bracketed by CUDA
- * events on the handle's stream.  skipconv_profile resets both. */
+ * convolution of the open blocks (either path), 3 y refresh, 4 the fused step
+ * (all of 0-2 in one launch).  Launch counts are always kept; with enable = 1
+ * each launch is also bracketed by CUDA events on the handle's stream.
+ * skipconv_profile resets both. */
+#define SKIPCONV_PROFILE_KINDS 5
 SKIPCONV_API int skipconv_profile(skipconv_handle h, int enable);
-/* Synchronise the stream and report, per kernel kind (arrays of 4), the
- * launches and the summed event-timed milliseconds since skipconv_profile
- * (milliseconds are 0 unless timing was enabled). */
+/* Synchronise the stream and report, per kernel kind (arrays of
+ * SKIPCONV_PROFILE_KINDS), the launches and the summed event-timed
+ * milliseconds since skipconv_profile (milliseconds are 0 unless timing was
+ * enabled). */
 SKIPCONV_API int skipconv_profile_read(skipconv_handle h, long long* launches, double* ms);
 
 /* Largest n_streams*h*w that skipconv_gate_noalloc accepts: its static device

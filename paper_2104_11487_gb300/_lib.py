@@ -19,7 +19,8 @@ SKIPCONV_ERR_DEVICE = -6
 GATE_INPUT_MEAN, GATE_INPUT_SUM, GATE_OUTPUT = 0, 1, 2
 F32, BF16 = 0, 1
 ACT_NONE, ACT_RELU, ACT_SILU = 0, 1, 2
-PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE = 0, 1, 2
+PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE, PATH_TENSOR_CORE_SEPARATE = 0, 1, 2, 3
+PROFILE_KINDS = 5   # gate_pixel, gate_block, conv, y_refresh, fused step
 
 # Every function the header declares, with its ctypes signature.
 SIGNATURES = {
@@ -51,7 +52,7 @@ class Params(ctypes.Structure):
 
 class Info(ctypes.Structure):
     _fields_ = [(n, c_int) for n in ("ho", "wo", "nby", "nbx", "conv_path", "num_sms")] + [
-        ("state_bytes", ctypes.c_size_t)]
+        ("state_bytes", ctypes.c_size_t), ("fused", c_int)]
 
 
 class SkipConvError(RuntimeError):

@@ -119,7 +119,7 @@ static void free_buffers(Layer* L)
 {
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
-                    L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage};
+                    L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);
@@ -158,7 +158,7 @@ int validate(const skipconv_params* p)
         return set_error("unknown dtype %d", p->dtype), SKIPCONV_ERR_INVALID;
     if (p->activation < SKIPCONV_ACT_NONE || p->activation > SKIPCONV_ACT_SILU)
         return set_error("unknown activation %d", p->activation), SKIPCONV_ERR_INVALID;
-    if (p->conv_path < SKIPCONV_PATH_AUTO || p->conv_path > SKIPCONV_PATH_TENSOR_CORE)
+    if (p->conv_path < SKIPCONV_PATH_AUTO || p->conv_path > SKIPCONV_PATH_TENSOR_CORE_SEPARATE)
         return set_error("unknown conv_path %d", p->conv_path), SKIPCONV_ERR_INVALID;
     const long long frame = (long long)p->n_streams * p->h * p->w;
     if (frame * p->c_in > (1LL << 40)) return set_error("frame too large"), SKIPCONV_ERR_INVALID;
@@ -233,7 +233,9 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
     // choose the convolution path
     const char* why = "";
     const bool tc_ok = conv_tc_supported(L.p, &why);
-    if (L.p.conv_path == SKIPCONV_PATH_TENSOR_CORE && !tc_ok) {
+    const bool want_tc = L.p.conv_path == SKIPCONV_PATH_TENSOR_CORE ||
+                         L.p.conv_path == SKIPCONV_PATH_TENSOR_CORE_SEPARATE;
+    if (want_tc && !tc_ok) {
         set_error("tensor-core path unsupported: %s", why);
         delete h;
         return SKIPCONV_ERR_UNSUPPORTED;
@@ -320,6 +322,25 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         e = conv_ws_prepare(L);
         L.tc_ws = e == cudaSuccess ? 1 : 0;
     }
+    // the whole step as one cooperative launch, unless the separate launches were asked for
+    if (e == cudaSuccess && L.tc_ws && L.p.conv_path != SKIPCONV_PATH_TENSOR_CORE_SEPARATE &&
+        step_fused_supported(L)) {
+        e = A.dev((void**)&L.sched, 16 * sizeof(int));
+        if (e == cudaSuccess) e = A.dev((void**)&L.pnorm, npix * sizeof(uint64_t));
+        if (e == cudaSuccess) e = A.dev((void**)&L.gtag, nblk * sizeof(uint32_t));
+        // tags start at 0, which no step uses
+        if (e == cudaSuccess) e = cudaMemsetAsync(L.pnorm, 0, npix * sizeof(uint64_t), L.stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(L.gtag, 0, nblk * sizeof(uint32_t), L.stream);
+        if (e == cudaSuccess) {
+            const cudaError_t pe = step_fused_prepare(L);
+            if (pe == cudaSuccess) {
+                L.fused = 1;
+            } else {
+                cudaGetLastError();   // not fatal: the separate launches serve this layer
+            }
+        }
+        L.state_bytes = A.bytes;
+    }
     if (e == cudaSuccess) {
         h->L.key = 1;
         st = skipconv_reset_state(h);
@@ -348,6 +369,7 @@ int skipconv_reset_state(skipconv_handle h)
     if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[0], 0, npix, L->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(L->chg[1], 0, npix, L->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(L->counters, 0, 64 * sizeof(int32_t), L->stream);
+    if (e == cudaSuccess && L->sched) e = cudaMemsetAsync(L->sched, 0, 16 * sizeof(int), L->stream);
     if (e == cudaSuccess) e = launch_reset_z(*L);
     if (e == cudaSuccess && L->y) e = cudaMemsetAsync(L->y, 0, (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * L->esize, L->stream);
     if (e != cudaSuccess) return status_of(e);
@@ -369,6 +391,15 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     // xbuf[cur] holds x_{t-1}; xbuf[nxt] holds x_{t-2} and receives x_t.
     // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
     const int force = (L->key || L->p.dense_mode) ? 1 : 0;
+    if (L->fused) {
+        const int slot = prof_begin(L, 4);
+        const cudaError_t e = launch_step_fused(*L, x_t, force);
+        prof_end(L, slot);
+        if (e != cudaSuccess) return status_of(e);
+        L->t += 1;
+        L->key = 0;
+        return SKIPCONV_OK;
+    }
     int slot = prof_begin(L, 0);
     cudaError_t e = launch_gate_pixels(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur], force);
     prof_end(L, slot);
@@ -479,6 +510,7 @@ int skipconv_get_info(skipconv_handle h, skipconv_info* info)
     info->nby = L->nby;
     info->nbx = L->nbx;
     info->conv_path = L->path;
+    info->fused = L->fused;
     info->num_sms = L->num_sms;
     info->state_bytes = L->state_bytes;
     return SKIPCONV_OK;
@@ -519,7 +551,7 @@ int skipconv_profile(skipconv_handle h, int enable)
     if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
     cudaError_t e = cudaStreamSynchronize(L->stream);
     if (e != cudaSuccess) return status_of(e);
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < SKIPCONV_PROFILE_KINDS; ++k) {
         L->launches[k] = 0;
         L->prof_ms[k] = 0.0;
     }
@@ -541,7 +573,7 @@ int skipconv_profile_read(skipconv_handle h, long long* launches, double* ms)
         L->prof_ms[L->prof_kind[i]] += t;
     }
     L->prof_n = 0;
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < SKIPCONV_PROFILE_KINDS; ++k) {
         if (launches) launches[k] = L->launches[k];
         if (ms) ms[k] = L->prof_ms[k];
     }

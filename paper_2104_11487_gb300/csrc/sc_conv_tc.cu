@@ -82,7 +82,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
                const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_z, const TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* smem = ptx::align_smem_1024(smem_raw);
     const int XB = x_tile_bytes(a.HH, a.WW);
     uint8_t* sA = smem;
     uint8_t* sX = smem + TC_ASTAGES * TC_ABYTES;

@@ -46,12 +46,12 @@ struct Layer {
     int* err_dev;
 
     // profiling (host): launch counts per kernel kind, optional event pairs
-    long long launches[4];
+    long long launches[SKIPCONV_PROFILE_KINDS];
     int prof_on;
     int prof_n, prof_cap;
     cudaEvent_t* prof_ev;   // 2 * prof_cap events
     int* prof_kind;
-    double prof_ms[4];
+    double prof_ms[SKIPCONV_PROFILE_KINDS];
 
     // recurrence bookkeeping (host)
     long long t;            // steps since reset (selects the ping-pong buffers)
@@ -65,6 +65,13 @@ struct Layer {
     CUtensorMap tmap_xrow[2];  // weight-stationary kernel: 128-byte-row halo boxes of the state frames
     int tc_z_tma;           // 1: the z tensor map below is valid (c_out multiple of 4)
     CUtensorMap tmap_z;
+
+    // fused step kernel (sc_step_fused.cu)
+    int fused;              // 1: the whole step is one cooperative launch
+    int* sched;             // fused step: grid abort flag (16 ints reserved)
+    uint64_t* pnorm;        // fused step: per pixel (epoch << 32) | fp32 norm
+    uint32_t* gtag;         // fused step: per gate block (epoch << 1) | open
+    uint32_t epoch;         // fused step: tag of the last launched step
 };
 
 // ------------------------------------------------------------------ launchers
@@ -95,6 +102,12 @@ cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, 
 bool conv_ws_supported(const Layer& L);
 cudaError_t conv_ws_prepare(Layer& L);
 cudaError_t launch_conv_ws(const Layer& L, const void* x_t, int prev_index);
+
+// Fused step (sc_step_fused.cu): gate passes 1-2 and the weight-stationary
+// convolution in one persistent cooperative launch, pipelined over streams.
+bool step_fused_supported(const Layer& L);
+cudaError_t step_fused_prepare(Layer& L);
+cudaError_t launch_step_fused(Layer& L, const void* x_t, int force);
 
 // Driver entry point for tensor-map encoding (resolved once through the runtime).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

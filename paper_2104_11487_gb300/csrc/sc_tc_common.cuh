@@ -41,5 +41,8 @@ __device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
 // Tensor maps (sc_conv_tc.cu): halo boxes of a frame, and the z state.
 bool tc_encode_x_map(CUtensorMap* m, const void* base, const Layer& L, bool five_d);
 bool tc_encode_z_map(CUtensorMap* m, const Layer& L);
+// Halo rows for the weight-stationary kernels (sc_conv_ws.cu): 4-D boxes of
+// 64 channels (128 bytes) x (8+k_w-1) x (8+k_h-1) pixels of one stream.
+bool encode_xrow_map(CUtensorMap* m, const void* base, const Layer& L);
 
 }  // namespace sc

@@ -91,14 +91,17 @@ def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_
 
 
 def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
-                     reset_at=(), emit_y=False):
+                     reset_at=(), emit_y=False, expect_fused=None):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
-    both sides; returns the Compare record."""
+    both sides; returns the Compare record and the conv path used.
+    expect_fused: None, or whether the layer must run as one fused launch."""
     import oracle
     ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode)
     gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y)
     cmp = Compare(spec, dtype, name)
     try:
+        if expect_fused is not None:
+            assert gl.info.fused == int(expect_fused), "%s: fused=%d" % (name, gl.info.fused)
         for t, f in enumerate(frames):
             if t in reset_at:
                 ref.reset()

@@ -10,7 +10,10 @@ from oracle import GATE_INPUT_SUM, GATE_OUTPUT, LayerSpec
 
 pytestmark = pytest.mark.gpu
 
-AUTO, CUDA_CORE, TENSOR_CORE = 0, 1, 2
+AUTO, CUDA_CORE, TENSOR_CORE, SEPARATE = 0, 1, 2, 3
+# AUTO runs these bf16 8x8-block layers as one fused launch per step; SEPARATE
+# forces the gate and the tensor-core convolution into their own launches.
+FUSED = {AUTO: True, SEPARATE: False, CUDA_CORE: False}
 
 
 def spec_of(wl, li=0, **kw):
@@ -36,11 +39,11 @@ def test_c0_fp32_pixel_gates():
     assert cmp.max_err <= 1e-4
 
 
-@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
 def test_c1_bf16_8x8_blocks(path):
     wl = synth.make_workload("c1")
     cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
-                                 conv_path=path, name="c1")
+                                 conv_path=path, name="c1", expect_fused=FUSED[path])
     assert cmp.frames == 16
 
 
@@ -66,32 +69,33 @@ def test_c3_mbconv_stack_teacher_forced():
 
 
 @pytest.mark.parametrize("density", [0.0, 0.1, 0.5, 1.0])
-@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
 def test_c4_density_small(density, path):
     """c4's generator at a small size (2 streams, 32x40, 64 channels), 32 frames."""
     wl = synth.make_workload("c4", density=density, T=32, n=2, h=32, w=40, c=64)
     cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
-                                 conv_path=path, name="c4-small d=%g" % density)
+                                 conv_path=path, name="c4-small d=%g" % density, expect_fused=FUSED[path])
     assert cmp.frames == 32
 
 
-@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
 def test_ragged_tail_and_several_tiles(path):
     """Frame sizes that are not multiples of the block (ragged edge blocks)."""
-    frames = synth.round_to_bf16(synth.moving_squares_video(77, 6, 100, 76, 32, n_squares=4, size=12))
+    frames = synth.round_to_bf16(synth.moving_squares_video(77, 6, 100, 76, 64, n_squares=4, size=12))
     rng = np.random.default_rng(78)
-    w = synth.he_weights(rng, 48, 32, 3, bf16=True)
+    w = synth.he_weights(rng, 48, 64, 3, bf16=True)
     b = synth.round_to_bf16(rng.standard_normal(48).astype(np.float32) * 0.1)
-    spec = LayerSpec(n=1, c_in=32, c_out=48, h=100, w=76, k=3, block=8, eps=0.05)
-    cmp, _ = run_single_layer(spec, w, b, [f[None] for f in frames], "bf16", conv_path=path, name="ragged")
+    spec = LayerSpec(n=1, c_in=64, c_out=48, h=100, w=76, k=3, block=8, eps=0.05)
+    cmp, _ = run_single_layer(spec, w, b, [f[None] for f in frames], "bf16", conv_path=path, name="ragged",
+                              expect_fused=FUSED[path])
     assert cmp.frames == 6
 
 
-@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
 def test_dense_mode_is_dense_conv(path):
     wl = synth.make_workload("c1", T=4)
     cmp, _ = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
-                              dense_mode=True, conv_path=path, name="dense")
+                              dense_mode=True, conv_path=path, name="dense", expect_fused=FUSED[path])
     assert cmp.frames == 4
 
 
@@ -132,10 +136,12 @@ def test_zero_residual_keeps_state_bitwise():
         gl.close()
 
 
-def test_c4_full_size_sampled():
+@pytest.mark.parametrize("path", [AUTO, SEPARATE])
+def test_c4_full_size_sampled(path):
     """The bench's configuration (8 streams of 128x128x256, 8x8 blocks, 10%
-    block density, 32 frames): full masks and lists every frame, z at sampled
-    locations (the oracle keeps only those)."""
+    block density, 32 frames; AUTO is the bench's fused launch): full masks
+    and lists every frame, z at sampled locations (the oracle keeps only
+    those)."""
     import oracle
     from harness import gpu_layer
     wl = synth.make_workload("c4", density=0.10, T=32)
@@ -144,9 +150,10 @@ def test_c4_full_size_sampled():
     samples = np.stack([rng.integers(0, spec.n, 192), rng.integers(0, spec.ho, 192),
                         rng.integers(0, spec.wo, 192)], axis=1).astype(np.int32)
     ref = oracle.SampledOracleLayer(spec, wl.weights[0], samples, wl.biases[0])
-    gl = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16")
+    gl = gpu_layer(spec, wl.weights[0], wl.biases[0], "bf16", conv_path=path)
     cmp = Compare(spec, "bf16", "c4-full")
     try:
+        assert gl.info.fused == int(FUSED[path])
         for t, f in wl.frames:
             forced = ref.key
             mask_ref = ref.step(f)
