@@ -44,10 +44,14 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--density", type=float, default=0.10)
+    ap.add_argument("--path", choices=("fused", "separate"), default="fused",
+                    help="fused: one launch per step (default); separate: gate passes and convolution launched apart")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-soak", action="store_true",
+                    help="skip the untimed steps around the timed region (for profiler runs)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
 
@@ -154,6 +158,20 @@ def flush_l2(buf):
     buf.view(-1, 4096).amax(dim=1)
 
 
+def soak(layer, frames, flush, seconds, torch):
+    """Untimed steps of the same workload (with the same L2 flush between
+    steps) for about `seconds`, so that the clock sampler sees the GPU under
+    this load for long enough: the timed region itself lasts milliseconds."""
+    t_end = time.perf_counter() + seconds
+    i = 0
+    while time.perf_counter() < t_end:
+        for _ in range(20):
+            flush_l2(flush)
+            layer.step(frames[1 + i % (len(frames) - 1)])
+            i += 1
+        torch.cuda.synchronize()
+
+
 def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
     """Key frame + `warmup` untimed steps, then `steps` timed steps with an L2
     flush between them (outside the events).  Returns per-step ms, per-kernel
@@ -184,10 +202,14 @@ def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
     return ms, launches, kms, counts, key_ms
 
 
-def make_layer(wl, torch, dense_mode=False):
+CONV_PATH = {"fused": 0, "separate": 3}   # AUTO (one fused launch per step) / TENSOR_CORE_SEPARATE
+
+
+def make_layer(wl, torch, dense_mode=False, path="fused"):
     from paper_2104_11487_gb300 import SkipConvLayer
     return SkipConvLayer(N_STREAMS, C, C, H, W, k=K, stride=1, pad=1, block=BLOCK, eps=EPS, dtype="bf16",
-                         dense_mode=dense_mode, weights=torch.from_numpy(wl.weights[0]), bias=None)
+                         dense_mode=dense_mode, conv_path=CONV_PATH[path],
+                         weights=torch.from_numpy(wl.weights[0]), bias=None)
 
 
 PROFILE_FILES = {"gate_pixel": ("gate_pixel", ("sc_gate.cu",)), "gate_block": ("gate_block", ("sc_gate.cu",)),
@@ -294,16 +316,22 @@ def main():
     n_frames = args.warmup + args.steps + 1
     wl, frames, changed = device_frames(args.density, n_frames, rank, torch)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    layer = make_layer(wl, torch)
+    layer = make_layer(wl, torch, path=args.path)
     info = skipconv_get_info(layer.handle)
 
     # 1) headline: timed steps, no per-kernel events
     clocks = Clocks(local)
     barrier()
     clocks.start()
+    if not args.no_soak:
+        soak(layer, frames, flush, 0.5, torch)
+    barrier()
     ms, launches, _, _, key_ms = run_layer_timed(layer, frames, args.warmup, args.steps, flush, torch)
     barrier()
+    if not args.no_soak:
+        soak(layer, frames, flush, 0.5, torch)
     clk = clocks.stop()
+    clk["window"] = "every 100 ms over the timed steps and 0.5 s of the same steps before and after"
     total_ms = max_over_ranks(sum(ms))
     ms_per_step = total_ms / args.steps
     value = world * N_STREAMS * args.steps / (total_ms / 1e3)
@@ -385,11 +413,11 @@ def main():
         dense_ms = None
         for d in (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00):
             wl_d, fr_d, ch_d = device_frames(d, args.warmup + args.sweep_steps + 1, rank, torch)
-            lay_d = make_layer(wl_d, torch)
+            lay_d = make_layer(wl_d, torch, path=args.path)
             ms_d, _, _, cnt_d, _ = run_layer_timed(lay_d, fr_d, args.warmup, args.sweep_steps, flush, torch,
                                                    profile=True)
             if d == 0.10:
-                lay_dense = make_layer(wl_d, torch, dense_mode=True)
+                lay_dense = make_layer(wl_d, torch, dense_mode=True, path=args.path)
                 ms_dn, _, _, _, _ = run_layer_timed(lay_dense, fr_d, args.warmup, args.sweep_steps, flush, torch)
                 dense_ms = statistics.median(ms_dn)
                 lay_dense.close()
