@@ -44,6 +44,12 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--density", type=float, default=0.10)
+    ap.add_argument("--gate", choices=("input", "output"), default="input",
+                    help="input: Input-Norm gate (Eq. 5, mean over the support); output: Output-Norm gate (Eq. 7)")
+    ap.add_argument("--key-interval", type=int, default=0,
+                    help="a key frame every K steps (Table 4's periodic reset); 0: none after the first")
+    ap.add_argument("--drift", action="store_true",
+                    help="add a drift report: Skip-Conv z~ against the dense closed form for several key intervals")
     ap.add_argument("--path", choices=("fused", "separate"), default="fused",
                     help="fused: one launch per step (default); separate: gate passes and convolution launched apart")
     ap.add_argument("--no-sweep", action="store_true")
@@ -58,11 +64,12 @@ def parse():
     return ap.parse_args()
 
 
-def workload_config(density, flushed=True):
+def workload_config(density, flushed=True, gate="input", key_interval=0):
     return {"workload": "c4: 3x3 Skip-Conv 256->256, %d streams x %dx%d, bf16 (fp32 accum), %dx%d blocks, "
                         "eps %.2g, %g%% block density" % (N_STREAMS, H, W, BLOCK, BLOCK, EPS, density * 100),
             "streams": N_STREAMS, "h": H, "w": W, "c_in": C, "c_out": C, "k": K, "block": BLOCK, "eps": EPS,
-            "gate": "input-norm (mean over support)", "density": density,
+            "gate": {"input": "input-norm (mean over support)", "output": "output-norm (Eq. 7)"}[gate],
+            "key_interval": key_interval, "density": density,
             "l2": ("flushed between timed steps (256 MiB written, then read back)" if flushed else
                    "not flushed: each step streams two 64 MiB frames per step in stream order, more than the 129 MB L2"),
             "parallelism": "replicas"}
@@ -211,11 +218,14 @@ def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
 CONV_PATH = {"fused": 0, "separate": 3}   # AUTO (one fused launch per step) / TENSOR_CORE_SEPARATE
 
 
-def make_layer(wl, torch, dense_mode=False, path="fused"):
+GATES = {"input": 0, "output": 2}         # Input-Norm (mean), Output-Norm
+
+
+def make_layer(wl, torch, dense_mode=False, path="fused", gate="input", key_interval=0):
     from paper_2104_11487_gb300 import SkipConvLayer
     return SkipConvLayer(N_STREAMS, C, C, H, W, k=K, stride=1, pad=1, block=BLOCK, eps=EPS, dtype="bf16",
-                         dense_mode=dense_mode, conv_path=CONV_PATH[path],
-                         weights=torch.from_numpy(wl.weights[0]), bias=None)
+                         dense_mode=dense_mode, conv_path=CONV_PATH[path], gate=GATES[gate],
+                         key_interval=key_interval, weights=torch.from_numpy(wl.weights[0]), bias=None)
 
 
 PROFILE_FILES = {"gate_pixel": ("gate_pixel", ("sc_gate.cu",)), "gate_block": ("gate_block", ("sc_gate.cu",)),
@@ -253,6 +263,52 @@ def traffic_from_profiles(kernel):
         if line.startswith("source_sha256:") and line.split(":", 1)[1].strip().split()[0] == digest:
             source_ok = True
     return traffic if source_ok else None
+
+
+# ----------------------------------------------------------- drift report
+def drift_report(torch, intervals=(0, 4, 8, 16), T=32):
+    """Skip-Conv z~ against the dense closed form z_t = w * x_t + b (a layer
+    that is reset at every step) on the moving-squares workload with
+    N(0, 0.01) noise (1 x 128 x 128 x 64 bf16, 8x8 blocks, eps 0.05): gates
+    skip the small residuals, whose effect on z~ persists until the next key
+    frame (Table 4).  Per key interval K: the largest and mean max-abs drift
+    relative to RMS(z_t) over the frames, and the mean open-block density."""
+    import synth
+    from paper_2104_11487_gb300 import SkipConvLayer
+    wl = synth.make_workload("c1", T=T)
+    L = wl.layers[0]
+    frames = [torch.from_numpy(np.ascontiguousarray(wl.frames[t])).cuda().to(torch.bfloat16) for t in range(T)]
+
+    def layer(k):
+        return SkipConvLayer(wl.n, L.c_in, L.c_out, wl.h, wl.w, k=L.k, stride=L.stride, pad=L.pad, block=L.block,
+                             eps=L.eps, dtype="bf16", key_interval=k, weights=torch.from_numpy(wl.weights[0]),
+                             bias=None if wl.biases[0] is None else torch.from_numpy(wl.biases[0]))
+    ref = layer(1)
+    lays = {k: layer(k) for k in intervals}
+    drift = {k: [] for k in intervals}
+    p99 = {k: [] for k in intervals}
+    dens = {k: [] for k in intervals}
+    nblk = wl.n * lays[intervals[0]].info.nby * lays[intervals[0]].info.nbx
+    for x in frames:
+        ref.step(x)
+        zr = ref.z().double()
+        rms = float(zr.pow(2).mean().sqrt())
+        for k, lay in lays.items():
+            lay.step(x)
+            err = (lay.z().double() - zr).abs().flatten()
+            drift[k].append(float(err.max()) / rms)
+            p99[k].append(float(torch.kthvalue(err.cpu(), int(0.99 * err.numel())).values) / rms)
+            dens[k].append(lay.gate()[2] / nblk)
+    out = {}
+    for k in intervals:
+        d = drift[k][1:]          # frame 0 is a key frame everywhere
+        out[str(k)] = {"max_rel_drift": max(d), "mean_rel_drift": sum(d) / len(d),
+                       "p99_rel_drift": max(p99[k][1:]),
+                       "mean_block_density": sum(dens[k][1:]) / (T - 1)}
+    for lay in list(lays.values()) + [ref]:
+        lay.close()
+    return {"workload": "moving squares + N(0,0.01) noise, 1 x 128x128x64 bf16, 3x3, 8x8 blocks, eps 0.05, %d frames" % T,
+            "reference": "the same layer reset at every step (z_t = w * x_t + b)", "key_interval": out}
 
 
 # ----------------------------------------------------------- CPU oracle
@@ -322,7 +378,7 @@ def main():
     n_frames = args.warmup + args.steps + 1
     wl, frames, changed = device_frames(args.density, n_frames, rank, torch)
     flush = None if args.no_flush else torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    layer = make_layer(wl, torch, path=args.path)
+    layer = make_layer(wl, torch, path=args.path, gate=args.gate, key_interval=args.key_interval)
     info = skipconv_get_info(layer.handle)
 
     # 1) headline: timed steps, no per-kernel events
@@ -382,7 +438,8 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded block-perturbation video)",
-            "config": workload_config(args.density, flushed=not args.no_flush),
+            "config": workload_config(args.density, flushed=not args.no_flush, gate=args.gate,
+                                      key_interval=args.key_interval),
             "conv_path": {1: "cuda-core", 2: "tensor-core"}.get(info.conv_path),
             "step_launches": "one fused launch" if info.fused else "separate gate and convolution launches",
             "active_blocks_per_step": active, "block_density_measured": active / (N_STREAMS * (H // BLOCK) ** 2),
@@ -419,11 +476,11 @@ def main():
         dense_ms = None
         for d in (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00):
             wl_d, fr_d, ch_d = device_frames(d, args.warmup + args.sweep_steps + 1, rank, torch)
-            lay_d = make_layer(wl_d, torch, path=args.path)
+            lay_d = make_layer(wl_d, torch, path=args.path, gate=args.gate, key_interval=args.key_interval)
             ms_d, _, _, cnt_d, _ = run_layer_timed(lay_d, fr_d, args.warmup, args.sweep_steps, flush, torch,
                                                    profile=True)
             if d == 0.10:
-                lay_dense = make_layer(wl_d, torch, dense_mode=True, path=args.path)
+                lay_dense = make_layer(wl_d, torch, dense_mode=True, path=args.path, gate=args.gate)
                 ms_dn, _, _, _, _ = run_layer_timed(lay_dense, fr_d, args.warmup, args.sweep_steps, flush, torch)
                 dense_ms = statistics.median(ms_dn)
                 lay_dense.close()
@@ -444,6 +501,8 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_oracle_sample(args.cpu_seconds, args.density)
     layer.close()
+    if args.drift and rank == 0:
+        line["drift_vs_dense"] = drift_report(torch)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:

@@ -98,6 +98,9 @@ typedef struct {
     int emit_y;        /* 1: keep y = act(z [+ shortcut]) in dtype for the next layer */
     int dense_mode;    /* 1: every gate open (in-library dense reference)           */
     int conv_path;     /* skipconv_path                                             */
+    int key_interval;  /* > 0: every key_interval-th step after a key frame is a key
+                          frame again (Table 4's periodic reset: x_{t-1} = 0,
+                          z = bias, whole frame); 0: only after create or reset */
 } skipconv_params;
 
 /* Create a layer.  Copies and repacks the weights (device pointer, OIHW,
@@ -116,7 +119,9 @@ SKIPCONV_API int skipconv_create(const skipconv_params* params, const void* weig
  * Enqueued on the handle's stream. */
 SKIPCONV_API int skipconv_reset_state(skipconv_handle h);
 
-/* One Skip-Conv step (Eq. 2, 5/7, 3).  x_t: device frame [n][h][w][c_in] in
+/* One Skip-Conv step (Eq. 2, 5/7, 3); a key frame when the handle was just
+ * created or reset, or when params.key_interval steps have passed since the
+ * last key frame (then the reset is enqueued first).  x_t: device frame [n][h][w][c_in] in
  * dtype, 16-byte aligned.  shortcut: NULL, or a device tensor
  * [n][ho][wo][c_out] in dtype added to z before the activation when y is
  * kept (then y is refreshed over the whole frame).  Updates z in place at the

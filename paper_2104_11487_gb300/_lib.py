@@ -47,7 +47,7 @@ SIGNATURES = {
 class Params(ctypes.Structure):
     _fields_ = [(n, c_int) for n in ("n_streams", "c_in", "c_out", "h", "w", "k_h", "k_w", "stride", "pad",
                                      "groups", "block")] + [("eps", c_float)] + [
-        (n, c_int) for n in ("gate", "dtype", "activation", "emit_y", "dense_mode", "conv_path")]
+        (n, c_int) for n in ("gate", "dtype", "activation", "emit_y", "dense_mode", "conv_path", "key_interval")]
 
 
 class Info(ctypes.Structure):

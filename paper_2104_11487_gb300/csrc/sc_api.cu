@@ -152,6 +152,7 @@ int validate(const skipconv_params* p)
     if (p->h + 2 * p->pad < p->k_h || p->w + 2 * p->pad < p->k_w)
         return set_error("kernel larger than the padded frame"), SKIPCONV_ERR_INVALID;
     if (!(p->eps >= 0.f)) return set_error("eps must be >= 0"), SKIPCONV_ERR_INVALID;
+    if (p->key_interval < 0) return set_error("key_interval must be >= 0"), SKIPCONV_ERR_INVALID;
     if (p->gate < SKIPCONV_GATE_INPUT_MEAN || p->gate > SKIPCONV_GATE_OUTPUT)
         return set_error("unknown gate %d", p->gate), SKIPCONV_ERR_INVALID;
     if (p->dtype != SKIPCONV_F32 && p->dtype != SKIPCONV_BF16)
@@ -387,6 +388,10 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
         return set_error("x_t and shortcut must be 16-byte aligned"), SKIPCONV_ERR_INVALID;
     if (shortcut && !L->y) return set_error("shortcut given but the layer keeps no y (emit_y = 0)"), SKIPCONV_ERR_INVALID;
     if (int st = check_device_word(L)) return st;
+    if (L->p.key_interval > 0 && !L->key && L->since_key >= L->p.key_interval) {
+        const int st = skipconv_reset_state(h);   // periodic key frame (Table 4)
+        if (st != SKIPCONV_OK) return st;
+    }
     const int cur = (int)(L->t & 1), nxt = cur ^ 1;
     // xbuf[cur] holds x_{t-1}; xbuf[nxt] holds x_{t-2} and receives x_t.
     // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
@@ -396,6 +401,7 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
         const cudaError_t e = launch_step_fused(*L, x_t, force);
         prof_end(L, slot);
         if (e != cudaSuccess) return status_of(e);
+        L->since_key = force && L->key ? 1 : L->since_key + 1;
         L->t += 1;
         L->key = 0;
         return SKIPCONV_OK;
@@ -421,6 +427,7 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
         prof_end(L, slot);
     }
     if (e != cudaSuccess) return status_of(e);
+    L->since_key = force && L->key ? 1 : L->since_key + 1;
     L->t += 1;
     L->key = 0;
     return SKIPCONV_OK;

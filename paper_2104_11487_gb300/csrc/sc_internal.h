@@ -56,6 +56,7 @@ struct Layer {
     // recurrence bookkeeping (host)
     long long t;            // steps since reset (selects the ping-pong buffers)
     int key;                // next step is a key frame
+    long long since_key;    // steps since the last key frame, that one included
 
     // tensor-core path: prebuilt TMA descriptors of the two x_{t-1} buffers and the weights
     int tc_x5d;             // 1: halo tiles as one 5-D TMA box per channel chunk; 0: 4-D boxes per 8 channels

@@ -119,13 +119,13 @@ class SkipConvLayer:
 
     def __init__(self, n_streams, c_in, c_out, h, w, k=3, stride=1, pad=1, groups=1, block=8, eps=0.05,
                  gate=GATE_INPUT_MEAN, dtype="bf16", activation=ACT_NONE, emit_y=False, dense_mode=False,
-                 conv_path=PATH_AUTO, weights=None, bias=None, stream=None):
+                 conv_path=PATH_AUTO, weights=None, bias=None, stream=None, key_interval=0):
         import torch
         self.torch = torch
         self.dtype = torch.bfloat16 if dtype == "bf16" else torch.float32
         self.params = Params(n_streams, c_in, c_out, h, w, k, k, stride, pad, groups, block, float(eps), gate,
                              BF16 if dtype == "bf16" else F32, activation, int(bool(emit_y)), int(bool(dense_mode)),
-                             conv_path)
+                             conv_path, int(key_interval))
         dev = torch.device("cuda", torch.cuda.current_device())
         w_t = torch.as_tensor(weights).to(device=dev, dtype=self.dtype).contiguous()
         b_t = None if bias is None else torch.as_tensor(bias).to(device=dev, dtype=torch.float32).contiguous()

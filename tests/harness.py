@@ -79,7 +79,7 @@ class Compare:
         self.frames += 1
 
 
-def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_path=0, gate=None):
+def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_path=0, gate=None, key_interval=0):
     import torch
     from paper_2104_11487_gb300 import SkipConvLayer
     wt = torch.from_numpy(np.ascontiguousarray(w, np.float32))
@@ -87,17 +87,21 @@ def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_
     return SkipConvLayer(spec.n, spec.c_in, spec.c_out, spec.h, spec.w, k=spec.k, stride=spec.stride, pad=spec.pad,
                          groups=spec.groups, block=spec.block, eps=spec.eps,
                          gate=spec.gate if gate is None else gate, dtype=dtype, activation=act, emit_y=emit_y,
-                         dense_mode=dense_mode, conv_path=conv_path, weights=wt, bias=bt)
+                         dense_mode=dense_mode, conv_path=conv_path, weights=wt, bias=bt, key_interval=key_interval)
 
 
 def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
-                     reset_at=(), emit_y=False, expect_fused=None):
+                     reset_at=(), emit_y=False, expect_fused=None, key_interval=0, ref_reset_at=()):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record and the conv path used.
-    expect_fused: None, or whether the layer must run as one fused launch."""
+    expect_fused: None, or whether the layer must run as one fused launch.
+    reset_at: frames before which both sides are reset; ref_reset_at: frames
+    before which only the oracle is reset (the GPU layer resets itself through
+    key_interval)."""
     import oracle
     ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode)
-    gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y)
+    gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y,
+                   key_interval=key_interval)
     cmp = Compare(spec, dtype, name)
     try:
         if expect_fused is not None:
@@ -106,6 +110,8 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
             if t in reset_at:
                 ref.reset()
                 gl.reset()
+            if t in ref_reset_at:
+                ref.reset()
             forced = ref.key or dense_mode
             score, mask_ref = ref.step(f)
             xt = to_device(f, dtype)

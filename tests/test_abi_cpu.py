@@ -46,7 +46,7 @@ def test_exported_symbols_are_only_the_abi():
 def test_params_struct_layout():
     from paper_2104_11487_gb300 import _lib
     # 11 ints, 1 float, 6 ints, no padding
-    assert ctypes.sizeof(_lib.Params) == 18 * 4
+    assert ctypes.sizeof(_lib.Params) == 19 * 4
     assert _lib.Params.eps.offset == 11 * 4
 
 

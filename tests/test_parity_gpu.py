@@ -118,6 +118,17 @@ def test_reset_mid_sequence_and_single_frame():
     assert cmp.frames == 1
 
 
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+def test_key_interval_resets_like_the_oracle(path):
+    """key_interval = 3: steps 3 and 6 are key frames (Table 4's periodic
+    reset), i.e. the oracle reset before frames 3 and 6."""
+    wl = synth.make_workload("c4", density=0.1, T=8, n=2, h=32, w=40, c=64)
+    cmp, _ = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16", conv_path=path,
+                              name="key interval", key_interval=3, ref_reset_at=(3, 6),
+                              expect_fused=FUSED[path])
+    assert cmp.frames == 8
+
+
 def test_zero_residual_keeps_state_bitwise():
     import torch
     from harness import gpu_layer
