@@ -27,6 +27,7 @@ _LIB_PATH = os.path.join(_HERE, "_build", "libskipconv_oracle.so")
 GATE_INPUT_MEAN = 0
 GATE_INPUT_SUM = 1
 GATE_OUTPUT = 2
+GATE_GUMBEL = 3
 ACT_NONE = 0
 ACT_RELU = 1
 ACT_SILU = 2
@@ -82,9 +83,11 @@ def lib():
         L.oc_block_gate.argtypes = [PP, _DP, ctypes.c_int, _UP]
         L.oc_dense_conv.argtypes = [PP, _DP, _DP, _DP, _DP]
         L.oc_reset.argtypes = [PP, _DP, _DP, _DP]
-        L.oc_step.argtypes = [PP, _DP, _DP, _DP, _DP, ctypes.c_int, _DP, _UP]
+        L.oc_gumbel_scores.argtypes = [PP, _DP, _DP, ctypes.c_double, _DP]
+        L.oc_step.argtypes = [PP, _DP, _DP, ctypes.c_double, _DP, _DP, _DP, ctypes.c_int, _DP, _UP]
         L.oc_step.restype = ctypes.c_long
-        L.oc_step_sampled.argtypes = [PP, _DP, _DP, _DP, ctypes.c_int, _IP, _DP, ctypes.c_int, _UP]
+        L.oc_step_sampled.argtypes = [PP, _DP, _DP, ctypes.c_double, _DP, _DP, ctypes.c_int, _IP, _DP, ctypes.c_int,
+                                      _UP]
         L.oc_step_sampled.restype = ctypes.c_long
         L.oc_round_bf16.argtypes = [ctypes.c_double]
         L.oc_round_bf16.restype = ctypes.c_double
@@ -160,6 +163,16 @@ def gate_scores(spec: LayerSpec, r, w=None) -> np.ndarray:
     return out
 
 
+def gumbel_scores(spec: LayerSpec, r, phi, phi_bias: float = 0.0) -> np.ndarray:
+    """Per-output-location Gumbel-gate score f(r; phi) (Eq. 8): a single-output-
+    channel convolution of r [n,h,w,c_in] with phi [c_in, k, k] plus phi_bias."""
+    r, phi = _f64(r), _f64(phi)
+    assert phi.shape == (spec.c_in, spec.k, spec.k)
+    out = np.empty((spec.n, spec.ho, spec.wo), np.float64)
+    lib().oc_gumbel_scores(ctypes.byref(spec.params()), _dp(r), _dp(phi), float(phi_bias), _dp(out))
+    return out
+
+
 def block_gate(spec: LayerSpec, score, force: bool = False) -> np.ndarray:
     score = _f64(score)
     out = np.empty((spec.n, spec.nby, spec.nbx), np.uint8)
@@ -194,10 +207,13 @@ def layer_output(z, shortcut=None, act: int = ACT_NONE, round_mode: int = 0) -> 
 class OracleLayer:
     """Stateful Skip-Conv layer: holds x_{t-1} and z~_{t-1} (Eq. 3) in double."""
 
-    def __init__(self, spec: LayerSpec, w, bias=None, dense_mode: bool = False):
+    def __init__(self, spec: LayerSpec, w, bias=None, dense_mode: bool = False, phi=None, phi_bias: float = 0.0):
         self.spec = spec
         self.w = _f64(w)
         assert self.w.shape == (spec.c_out, spec.c_in // spec.groups, spec.k, spec.k)
+        self.phi = None if phi is None else _f64(phi)          # Gumbel gate function (gate mode 3)
+        self.phi_bias = float(phi_bias)
+        assert spec.gate != GATE_GUMBEL or (self.phi is not None and self.phi.shape == (spec.c_in, spec.k, spec.k))
         self.bias = None if bias is None else _f64(bias)
         self.dense_mode = bool(dense_mode)
         self.x_prev = np.zeros((spec.n, spec.h, spec.w, spec.c_in), np.float64)
@@ -216,8 +232,8 @@ class OracleLayer:
         score = np.empty((s.n, s.ho, s.wo), np.float64)
         mask = np.empty((s.n, s.nby, s.nbx), np.uint8)
         f = self.key or self.dense_mode if force is None else force
-        rc = lib().oc_step(ctypes.byref(s.params()), _dp(self.w), _dp(x_t), _dp(self.x_prev),
-                           _dp(self.z), int(f), _dp(score), mask.ctypes.data_as(_UP))
+        rc = lib().oc_step(ctypes.byref(s.params()), _dp(self.w), _dp(self.phi), self.phi_bias, _dp(x_t),
+                           _dp(self.x_prev), _dp(self.z), int(f), _dp(score), mask.ctypes.data_as(_UP))
         if rc < 0:
             raise MemoryError("oracle step: allocation failed")
         self.key = False
@@ -230,9 +246,12 @@ class SampledOracleLayer:
     The gate is evaluated over the whole frame every step, so the sampled z
     values follow exactly the recurrence of the full state."""
 
-    def __init__(self, spec: LayerSpec, w, samples_nij, bias=None, dense_mode: bool = False):
+    def __init__(self, spec: LayerSpec, w, samples_nij, bias=None, dense_mode: bool = False, phi=None,
+                 phi_bias: float = 0.0):
         self.spec = spec
         self.w = _f64(w)
+        self.phi = None if phi is None else _f64(phi)
+        self.phi_bias = float(phi_bias)
         self.samples = np.ascontiguousarray(samples_nij, dtype=np.int32).reshape(-1, 3)
         self.bias = None if bias is None else _f64(bias)
         self.dense_mode = bool(dense_mode)
@@ -257,8 +276,8 @@ class SampledOracleLayer:
         x_t = _f64(x_t)
         mask = np.empty((s.n, s.nby, s.nbx), np.uint8)
         f = self.key or self.dense_mode if force is None else force
-        rc = lib().oc_step_sampled(ctypes.byref(s.params()), _dp(self.w), _dp(x_t), _dp(self.x_prev),
-                                   len(self.samples), self.samples.ctypes.data_as(_IP),
+        rc = lib().oc_step_sampled(ctypes.byref(s.params()), _dp(self.w), _dp(self.phi), self.phi_bias, _dp(x_t),
+                                   _dp(self.x_prev), len(self.samples), self.samples.ctypes.data_as(_IP),
                                    _dp(self.z), int(f), mask.ctypes.data_as(_UP))
         if rc < 0:
             raise MemoryError("oracle step: allocation failed")

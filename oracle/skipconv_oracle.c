@@ -38,11 +38,11 @@ typedef struct {
     int groups;
     int block;      /* b: edge of the b x b gate blocks (Sec. 3.2, structured sparsity) */
     int gate;       /* 0 input-norm, mean over the support; 1 input-norm, sum;
-                       2 output-norm (Eq. 7)                                 */
+                       2 output-norm (Eq. 7); 3 Gumbel gate (Eq. 8, inference) */
     double eps;
 } oc_params;
 
-enum { OC_GATE_INPUT_MEAN = 0, OC_GATE_INPUT_SUM = 1, OC_GATE_OUTPUT = 2 };
+enum { OC_GATE_INPUT_MEAN = 0, OC_GATE_INPUT_SUM = 1, OC_GATE_OUTPUT = 2, OC_GATE_GUMBEL = 3 };
 enum { OC_ACT_NONE = 0, OC_ACT_RELU = 1, OC_ACT_SILU = 2 };
 
 int oc_out_h(const oc_params* p) { return (p->h + 2 * p->pad - p->k_h) / p->stride + 1; }
@@ -138,6 +138,41 @@ void oc_gate_scores(const oc_params* p, const double* r, double w_l1, double* sc
             }
 }
 
+/* Gumbel-gate score at every output location (Eq. 8 at inference): the gate
+ * function f(r; phi) is a convolution of r with a single output channel and
+ * the layer's kernel size, stride and zero padding, plus its bias:
+ *   f(i,j) = phi_bias + sum_{c,kh,kw} phi[c][kh][kw] r[c, s i + kh - pad, s j + kw - pad].
+ * The gate round(sigmoid(f)) is 1 exactly when f > 0, i.e. the block gate
+ * below with eps = 0.  phi is [c_in][k_h][k_w]. */
+void oc_gumbel_scores(const oc_params* p, const double* r, const double* phi, double phi_bias, double* score)
+{
+    const int ho = oc_out_h(p), wo = oc_out_w(p);
+#ifdef _OPENMP
+#pragma omp parallel for collapse(2) schedule(static)
+#endif
+    for (int n = 0; n < p->n; ++n)
+        for (int i = 0; i < ho; ++i)
+            for (int j = 0; j < wo; ++j) {
+                double f = phi_bias;
+                for (int c = 0; c < p->c_in; ++c)
+                    for (int kh = 0; kh < p->k_h; ++kh)
+                        for (int kw = 0; kw < p->k_w; ++kw) {
+                            int y = p->stride * i + kh - p->pad;
+                            int x = p->stride * j + kw - p->pad;
+                            f += phi[((size_t)c * p->k_h + kh) * p->k_w + kw] * at_or_zero(p, r, n, y, x, c);
+                        }
+                score[((size_t)n * ho + i) * wo + j] = f;
+            }
+}
+
+/* The gate score of the layer's gate mode. */
+static void gate_scores_of(const oc_params* p, const double* w, const double* r, const double* phi, double phi_bias,
+                           double* score)
+{
+    if (p->gate == OC_GATE_GUMBEL) oc_gumbel_scores(p, r, phi, phi_bias, score);
+    else oc_gate_scores(p, r, p->gate == OC_GATE_OUTPUT ? oc_weight_l1(p, w) : 0.0, score);
+}
+
 /* Block gate (Sec. 3.2, structured sparsity): the pixel gate is
  * round(sigmoid(score - eps)), which is 1 exactly when score > eps; max-pooling
  * it with kernel and stride b opens a block when any of its locations is open.
@@ -201,11 +236,12 @@ void oc_reset(const oc_params* p, const double* bias, double* x_prev, double* z)
 
 /* One Skip-Conv step (Eq. 3):  z~_t = z~_{t-1} + g(r_t) (.) (w * r_t),
  * r_t = x_t - x_{t-1}; ungated locations keep z~_{t-1}; then x_{t-1} <- x_t.
+ * phi / phi_bias: the Gumbel gate's function (gate mode 3), else unused.
  * force = 1 opens every gate (key frame or dense mode).
  * score_out ([n][ho][wo]) and mask_out ([n][nby][nbx]) may be NULL.
  * Returns the number of open blocks, or -1 on allocation failure. */
-long oc_step(const oc_params* p, const double* w, const double* x_t, double* x_prev, double* z,
-             int force, double* score_out, unsigned char* mask_out)
+long oc_step(const oc_params* p, const double* w, const double* phi, double phi_bias, const double* x_t,
+             double* x_prev, double* z, int force, double* score_out, unsigned char* mask_out)
 {
     const int ho = oc_out_h(p), wo = oc_out_w(p);
     const int nby = oc_blocks_y(p), nbx = oc_blocks_x(p), b = p->block;
@@ -220,7 +256,7 @@ long oc_step(const oc_params* p, const double* w, const double* x_t, double* x_p
         return -1;
     }
     oc_residual(p, x_t, x_prev, r);
-    oc_gate_scores(p, r, p->gate == OC_GATE_OUTPUT ? oc_weight_l1(p, w) : 0.0, score);
+    gate_scores_of(p, w, r, phi, phi_bias, score);
     oc_block_gate(p, score, force, mask);
 #ifdef _OPENMP
 #pragma omp parallel for collapse(2) schedule(dynamic)
@@ -244,8 +280,8 @@ long oc_step(const oc_params* p, const double* w, const double* x_t, double* x_p
  * (z_samples is [n_samples][c_out], locations given as (n, i, j) triples).
  * The gate is evaluated over the whole frame exactly as in oc_step, so the
  * sampled z follows the same recurrence as the full one. */
-long oc_step_sampled(const oc_params* p, const double* w, const double* x_t, double* x_prev,
-                     int n_samples, const int* sample_nij, double* z_samples, int force,
+long oc_step_sampled(const oc_params* p, const double* w, const double* phi, double phi_bias, const double* x_t,
+                     double* x_prev, int n_samples, const int* sample_nij, double* z_samples, int force,
                      unsigned char* mask_out)
 {
     const int ho = oc_out_h(p), wo = oc_out_w(p);
@@ -261,7 +297,7 @@ long oc_step_sampled(const oc_params* p, const double* w, const double* x_t, dou
         return -1;
     }
     oc_residual(p, x_t, x_prev, r);
-    oc_gate_scores(p, r, p->gate == OC_GATE_OUTPUT ? oc_weight_l1(p, w) : 0.0, score);
+    gate_scores_of(p, w, r, phi, phi_bias, score);
     oc_block_gate(p, score, force, mask);
 #ifdef _OPENMP
 #pragma omp parallel for schedule(dynamic)

@@ -349,3 +349,76 @@ def test_sampled_layer_matches_full_layer():
         np.testing.assert_array_equal(samp.z, full.z[samples[:, 0], samples[:, 1], samples[:, 2]])
         x = x.copy()
         x[:, t:t + 3, 1:4] += rng.random((2, 3, 3, 4))
+
+
+# ------------------------------------------------------- Gumbel gate (Eq. 8)
+@pytest.mark.parametrize("si", range(len(SHAPES)))
+def test_gumbel_score_is_single_channel_conv(si):
+    """f(r; phi) is a convolution with one output channel and the layer's
+    kernel, stride and padding (plus its bias): torch's conv2d computes it."""
+    s = SHAPES[si]
+    spec = LayerSpec(n=s.n, c_in=s.c_in, c_out=s.c_out, h=s.h, w=s.w, k=s.k, stride=s.stride, pad=s.pad,
+                     groups=s.groups, block=s.block, eps=0.0, gate=oracle.GATE_GUMBEL)
+    rng = np.random.default_rng(300 + si)
+    r = rng.standard_normal((spec.n, spec.h, spec.w, spec.c_in))
+    phi = rng.standard_normal((spec.c_in, spec.k, spec.k))
+    bias = 0.37
+    ref = torch_conv(LayerSpec(n=spec.n, c_in=spec.c_in, c_out=1, h=spec.h, w=spec.w, k=spec.k, stride=spec.stride,
+                               pad=spec.pad), phi[None], r, [bias])[..., 0]
+    np.testing.assert_allclose(oracle.gumbel_scores(spec, r, phi, bias), ref, rtol=1e-12, atol=1e-12)
+
+
+def test_gumbel_zero_residual_and_linearity():
+    """r = 0 gives f = phi_bias everywhere (all gates open iff phi_bias > 0);
+    f - phi_bias is linear in r."""
+    spec = LayerSpec(n=1, c_in=3, c_out=2, h=7, w=6, k=3, block=2, eps=0.0, gate=oracle.GATE_GUMBEL)
+    rng = np.random.default_rng(310)
+    phi = rng.standard_normal((3, 3, 3))
+    zero = np.zeros((1, 7, 6, 3))
+    for b in (0.25, -0.25):
+        f = oracle.gumbel_scores(spec, zero, phi, b)
+        np.testing.assert_array_equal(f, np.full(f.shape, b))
+        assert oracle.block_gate(spec, f).all() == (b > 0) and oracle.block_gate(spec, f).any() == (b > 0)
+    r1, r2 = rng.standard_normal((2, 1, 7, 6, 3))
+    a = 1.7
+    lhs = oracle.gumbel_scores(spec, a * r1 + r2, phi, 0.0)
+    rhs = a * oracle.gumbel_scores(spec, r1, phi, 0.0) + oracle.gumbel_scores(spec, r2, phi, 0.0)
+    np.testing.assert_allclose(lhs, rhs, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("stride,block", [(1, 1), (2, 2), (1, 3)])
+def test_gumbel_step_is_masked_dense_update(stride, block):
+    """A Gumbel-gated step adds w * r exactly at the locations of blocks where
+    max f > 0 (round(sigmoid(f)) = 1), brute force on a tiny layer."""
+    spec = LayerSpec(n=1, c_in=2, c_out=3, h=6, w=5, k=3, stride=stride, pad=1, block=block, eps=0.0,
+                     gate=oracle.GATE_GUMBEL)
+    rng = np.random.default_rng(320 + stride + block)
+    w, b = rand_layer(rng, spec)
+    phi = rng.standard_normal((2, 3, 3))
+    phi_b = -0.5
+    frames = [rng.random((1, 6, 5, 2)) for _ in range(3)]
+    lay = OracleLayer(spec, w, b, phi=phi, phi_bias=phi_b)
+    z = torch_conv(spec, w, frames[0], b)
+    lay.step(frames[0])                              # key frame
+    np.testing.assert_allclose(lay.z, z, rtol=1e-12, atol=1e-12)
+    closed = 0
+    for t in (1, 2):
+        r = frames[t] - frames[t - 1]
+        f = torch_conv(LayerSpec(n=1, c_in=2, c_out=1, h=6, w=5, k=3, stride=stride, pad=1), phi[None], r,
+                       [phi_b])[..., 0]
+        ho, wo = f.shape[1:]
+        nby, nbx = -(-ho // block), -(-wo // block)
+        mask = np.zeros((1, nby, nbx), np.uint8)
+        for by in range(nby):
+            for bx in range(nbx):
+                mask[0, by, bx] = f[0, by * block:by * block + block, bx * block:bx * block + block].max() > 0
+        upd = torch_conv(spec, w, r)
+        for i in range(ho):
+            for j in range(wo):
+                if mask[0, i // block, j // block]:
+                    z[0, i, j] += upd[0, i, j]
+        _, m = lay.step(frames[t])
+        np.testing.assert_array_equal(m, mask)
+        closed += int((mask == 0).sum())
+        np.testing.assert_allclose(lay.z, z, rtol=1e-12, atol=1e-12)
+    assert closed > 0, "the case must close some gates"
