@@ -67,7 +67,12 @@ typedef enum {
 typedef enum {
     SKIPCONV_GATE_INPUT_MEAN = 0,  /* Eq. 5, l1 norm / (c_in*k_h*k_w) > eps    */
     SKIPCONV_GATE_INPUT_SUM = 1,   /* Eq. 5, l1 norm > eps                     */
-    SKIPCONV_GATE_OUTPUT = 2       /* Eq. 7, ||w||_1 * l1 norm > eps            */
+    SKIPCONV_GATE_OUTPUT = 2,      /* Eq. 7, ||w||_1 * l1 norm > eps            */
+    SKIPCONV_GATE_GUMBEL = 3       /* Eq. 8 at inference: f(r; phi) > eps, f a
+                                      one-output-channel conv of r with the layer's
+                                      kernel, stride and padding (eps = 0 is
+                                      round(sigmoid(f))); phi from
+                                      skipconv_set_gate_weights; k_h*k_w <= 9    */
 } skipconv_gate;
 
 typedef enum { SKIPCONV_F32 = 0, SKIPCONV_BF16 = 1 } skipconv_dtype;
@@ -135,6 +140,14 @@ SKIPCONV_API int skipconv_step(skipconv_handle h, const void* x_t, const void* s
  * may be NULL to skip the read-back), and synchronises the stream before
  * returning.  The first call allocates a device staging frame. */
 SKIPCONV_API int skipconv_step_host(skipconv_handle h, const void* x_t_host, float* z_out_host);
+
+/* The Gumbel gate's function (Eq. 8): phi_oihw, device float32
+ * [1][c_in][k_h][k_w] (one output channel, the layer's kernel size), and its
+ * bias.  Required before the first step of a SKIPCONV_GATE_GUMBEL layer; may
+ * be called again to replace phi.  Copies phi (through the host) and
+ * synchronises the stream.  Errors: INVALID (NULL handle or phi, a layer whose
+ * gate is not GUMBEL), CUDA. */
+SKIPCONV_API int skipconv_set_gate_weights(skipconv_handle h, const float* phi_oihw, float phi_bias);
 
 /* Synchronise the stream and free everything.  NULL is accepted. */
 SKIPCONV_API int skipconv_destroy(skipconv_handle h);

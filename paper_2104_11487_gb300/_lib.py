@@ -16,7 +16,7 @@ SKIPCONV_ERR_OOM = -4
 SKIPCONV_ERR_TIMEOUT = -5
 SKIPCONV_ERR_DEVICE = -6
 
-GATE_INPUT_MEAN, GATE_INPUT_SUM, GATE_OUTPUT = 0, 1, 2
+GATE_INPUT_MEAN, GATE_INPUT_SUM, GATE_OUTPUT, GATE_GUMBEL = 0, 1, 2, 3
 F32, BF16 = 0, 1
 ACT_NONE, ACT_RELU, ACT_SILU = 0, 1, 2
 PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE, PATH_TENSOR_CORE_SEPARATE = 0, 1, 2, 3
@@ -39,6 +39,7 @@ SIGNATURES = {
     "skipconv_profile": (c_int, [c_void_p, c_int]),
     "skipconv_profile_read": (c_int, [c_void_p, c_void_p, c_void_p]),
     "skipconv_gate_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "skipconv_set_gate_weights": (c_int, [c_void_p, c_void_p, c_float]),
     "skipconv_status_string": (ctypes.c_char_p, [c_int]),
     "skipconv_last_error": (ctypes.c_char_p, []),
 }

@@ -1,5 +1,6 @@
 // Host side of the Skip-Conv C ABI (include/skipconv.h): argument checks,
 // state allocation, weight repacking, and the per-step launch sequence
+//   step_fused (one launch), or
 //   gate_pixel -> gate_block -> conv (tensor-core or CUDA-core) [-> y_refresh]
 // all on the handle's stream, with no host synchronisation per step.
 #include <stdarg.h>
@@ -8,6 +9,7 @@
 #include <string.h>
 
 #include <new>
+#include <vector>
 
 #include "sc_internal.h"
 
@@ -119,7 +121,8 @@ static void free_buffers(Layer* L)
 {
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
-                    L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag};
+                    L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag,
+                    L->pix_taps, L->gphi};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);
@@ -153,7 +156,7 @@ int validate(const skipconv_params* p)
         return set_error("kernel larger than the padded frame"), SKIPCONV_ERR_INVALID;
     if (!(p->eps >= 0.f)) return set_error("eps must be >= 0"), SKIPCONV_ERR_INVALID;
     if (p->key_interval < 0) return set_error("key_interval must be >= 0"), SKIPCONV_ERR_INVALID;
-    if (p->gate < SKIPCONV_GATE_INPUT_MEAN || p->gate > SKIPCONV_GATE_OUTPUT)
+    if (p->gate < SKIPCONV_GATE_INPUT_MEAN || p->gate > SKIPCONV_GATE_GUMBEL)
         return set_error("unknown gate %d", p->gate), SKIPCONV_ERR_INVALID;
     if (p->dtype != SKIPCONV_F32 && p->dtype != SKIPCONV_BF16)
         return set_error("unknown dtype %d", p->dtype), SKIPCONV_ERR_INVALID;
@@ -167,6 +170,9 @@ int validate(const skipconv_params* p)
     const int wo = (p->w + 2 * p->pad - p->k_w) / p->stride + 1;
     const long long nblocks = (long long)p->n_streams * ((ho + p->block - 1) / p->block) * ((wo + p->block - 1) / p->block);
     if (nblocks >= (1LL << 31)) return set_error("too many gate blocks"), SKIPCONV_ERR_INVALID;
+    if (p->gate == SKIPCONV_GATE_GUMBEL &&
+        (p->k_h * p->k_w > 9 || (size_t)p->k_h * p->k_w * p->c_in * sizeof(float) > 48 * 1024))
+        return set_error("Gumbel gate: at most 9 taps and taps*c_in*4 <= 48 KiB"), SKIPCONV_ERR_UNSUPPORTED;
     if (p->c_in > gate_max_channels(p->dtype, false))
         return set_error("c_in above %d", gate_max_channels(p->dtype, false)), SKIPCONV_ERR_UNSUPPORTED;
     return SKIPCONV_OK;
@@ -265,6 +271,11 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
     if (e == cudaSuccess) e = A.dev((void**)&L.chg[0], npix);
     if (e == cudaSuccess) e = A.dev((void**)&L.chg[1], npix);
     if (e == cudaSuccess) e = A.dev((void**)&L.pix_l1, npix * sizeof(float));
+    if (e == cudaSuccess && L.p.gate == SKIPCONV_GATE_GUMBEL) {
+        const size_t taps = (size_t)L.p.k_h * L.p.k_w;
+        e = A.dev((void**)&L.pix_taps, npix * taps * sizeof(float));
+        if (e == cudaSuccess) e = A.dev((void**)&L.gphi, taps * L.p.c_in * sizeof(float));
+    }
     if (e == cudaSuccess) e = A.dev((void**)&L.mask, nblk);
     if (e == cudaSuccess) e = A.dev((void**)&L.list, nblk * sizeof(int32_t));
     if (e == cudaSuccess) e = A.dev((void**)&L.counters, 64 * sizeof(int32_t));
@@ -315,6 +326,7 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
     double thr;
     if (L.p.gate == SKIPCONV_GATE_INPUT_MEAN) thr = (double)L.p.eps * L.p.c_in * L.p.k_h * L.p.k_w;
     else if (L.p.gate == SKIPCONV_GATE_INPUT_SUM) thr = (double)L.p.eps;
+    else if (L.p.gate == SKIPCONV_GATE_GUMBEL) thr = (double)L.p.eps;
     else thr = w_l1 > 0.0 ? (double)L.p.eps / w_l1 : INFINITY;
     L.gate_thr = (float)thr;
 
@@ -388,6 +400,8 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
         return set_error("x_t and shortcut must be 16-byte aligned"), SKIPCONV_ERR_INVALID;
     if (shortcut && !L->y) return set_error("shortcut given but the layer keeps no y (emit_y = 0)"), SKIPCONV_ERR_INVALID;
     if (int st = check_device_word(L)) return st;
+    if (L->p.gate == SKIPCONV_GATE_GUMBEL && !L->gphi_set)
+        return set_error("Gumbel gate: call skipconv_set_gate_weights before the first step"), SKIPCONV_ERR_INVALID;
     if (L->p.key_interval > 0 && !L->key && L->since_key >= L->p.key_interval) {
         const int st = skipconv_reset_state(h);   // periodic key frame (Table 4)
         if (st != SKIPCONV_OK) return st;
@@ -406,12 +420,14 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
         L->key = 0;
         return SKIPCONV_OK;
     }
+    const bool gumbel = L->p.gate == SKIPCONV_GATE_GUMBEL;
     int slot = prof_begin(L, 0);
-    cudaError_t e = launch_gate_pixels(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur], force);
+    cudaError_t e = gumbel ? launch_gate_pixels_gumbel(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur])
+                           : launch_gate_pixels(*L, x_t, L->xbuf[cur], L->xbuf[nxt], L->chg[nxt], L->chg[cur], force);
     prof_end(L, slot);
     if (e == cudaSuccess) {
         slot = prof_begin(L, 1);
-        e = launch_gate_blocks(*L, force);
+        e = gumbel ? launch_gate_blocks_gumbel(*L, force) : launch_gate_blocks(*L, force);
         prof_end(L, slot);
     }
     if (e == cudaSuccess) {
@@ -430,6 +446,28 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     L->since_key = force && L->key ? 1 : L->since_key + 1;
     L->t += 1;
     L->key = 0;
+    return SKIPCONV_OK;
+}
+
+int skipconv_set_gate_weights(skipconv_handle h, const float* phi_oihw, float phi_bias)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!phi_oihw) return set_error("phi is NULL"), SKIPCONV_ERR_INVALID;
+    if (L->p.gate != SKIPCONV_GATE_GUMBEL)
+        return set_error("skipconv_set_gate_weights: the layer's gate is not SKIPCONV_GATE_GUMBEL"),
+               SKIPCONV_ERR_INVALID;
+    const int taps = L->p.k_h * L->p.k_w, C = L->p.c_in;
+    std::vector<float> src((size_t)taps * C), dst((size_t)taps * C);
+    cudaError_t e = cudaStreamSynchronize(L->stream);
+    if (e == cudaSuccess) e = cudaMemcpy(src.data(), phi_oihw, src.size() * sizeof(float), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return status_of(e);
+    for (int c = 0; c < C; ++c)            // [c][kh][kw] -> [tap][c]
+        for (int t = 0; t < taps; ++t) dst[(size_t)t * C + c] = src[(size_t)c * taps + t];
+    e = cudaMemcpy(L->gphi, dst.data(), dst.size() * sizeof(float), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return status_of(e);
+    L->gphi_bias = phi_bias;
+    L->gphi_set = 1;
     return SKIPCONV_OK;
 }
 

@@ -281,6 +281,126 @@ __global__ void __launch_bounds__(256) gate_block_kernel(const float* __restrict
     }
 }
 
+// Gumbel gate (Eq. 8 at inference), pass 1 of 2: one warp per input pixel.
+// The gate function f(r; phi) is a convolution of r with one output channel
+// and the layer's kernel; this pass forms, for each of the k_h*k_w taps t,
+// the pixel's partial product d_t = sum_c phi[t][c] r[c] (phi staged in shared
+// memory as [tap][channel]), plus the change flag and the state commit of the
+// norm pass.  Pass 2 sums the taps' partial products over each output
+// location's receptive field.
+constexpr int GUMBEL_MAX_TAPS = 9;
+
+template <typename T>
+__global__ void __launch_bounds__(256) gate_pixel_gumbel_kernel(
+    const T* __restrict__ xt, const T* __restrict__ xp, T* __restrict__ xn, const uint8_t* __restrict__ chg_prev,
+    uint8_t* __restrict__ chg_cur, const float* __restrict__ phi, float* __restrict__ taps_out, long long n_pix, int C,
+    int taps, int32_t* __restrict__ count_cur, int32_t* __restrict__ count_next)
+{
+    extern __shared__ float sphi[];  // [taps][C]
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        *count_cur = 0;
+        *count_next = 0;
+    }
+    for (int i = threadIdx.x; i < taps * C; i += blockDim.x) sphi[i] = phi[i];
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    for (long long pix = warp; pix < n_pix; pix += nwarps) {
+        float acc[GUMBEL_MAX_TAPS];
+#pragma unroll
+        for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) acc[t] = 0.f;
+        unsigned diff = 0;
+        for (int c = lane; c < C; c += 32) {
+            const T a = xt[pix * C + c], b = xp[pix * C + c];
+            const float r = to_f32(a) - to_f32(b);
+            if (sizeof(T) == 2)
+                diff |= (unsigned)(*reinterpret_cast<const uint16_t*>(&a) ^ *reinterpret_cast<const uint16_t*>(&b));
+            else
+                diff |= *reinterpret_cast<const uint32_t*>(&a) ^ *reinterpret_cast<const uint32_t*>(&b);
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t)
+                if (t < taps) acc[t] = fmaf(sphi[t * C + c], r, acc[t]);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) acc[t] += __shfl_xor_sync(0xffffffffu, acc[t], off);
+            diff |= __shfl_xor_sync(0xffffffffu, diff, off);
+        }
+        if (diff || chg_prev[pix])
+            for (int c = lane; c < C; c += 32) xn[pix * C + c] = xt[pix * C + c];
+        if (lane == 0) {
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t)
+                if (t < taps) taps_out[pix * taps + t] = acc[t];
+            chg_cur[pix] = diff ? 1 : 0;
+        }
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Gumbel gate, pass 2 of 2: one warp per gate block.  f at an output location
+// is phi_bias plus the partial products of the taps over its receptive field
+// (zero padding: out-of-frame taps add nothing); the block opens when its
+// largest f exceeds the threshold (eps; eps = 0 is round(sigmoid(f)) = 1).
+__global__ void __launch_bounds__(256) gate_block_gumbel_kernel(const float* __restrict__ taps_in,
+                                                                uint8_t* __restrict__ mask, int32_t* __restrict__ list,
+                                                                int32_t* __restrict__ count_cur, GateGeom g,
+                                                                float thr, float phi_bias, int force)
+{
+    __shared__ int flags[8];
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int taps = g.KH * g.KW;
+    const long long nblocks = (long long)g.n * g.nby * g.nbx;
+    const long long blk = (long long)blockIdx.x * 8 + wid;
+    int open = 0;
+    if (blk < nblocks) {
+        if (force) {
+            open = 1;
+        } else {
+            const int bx = (int)(blk % g.nbx);
+            const long long rest = blk / g.nbx;
+            const int by = (int)(rest % g.nby);
+            const int nn = (int)(rest / g.nby);
+            const float* Tn = taps_in + (size_t)nn * g.H * g.W * taps;
+            const int bh = min(g.b, g.Ho - by * g.b), bw = min(g.b, g.Wo - bx * g.b);
+            const int fy0 = by * g.b * g.stride - g.pad, fx0 = bx * g.b * g.stride - g.pad;
+            float best = -INFINITY;
+            for (int q = lane; q < bh * bw; q += 32) {
+                const int i = q / bw, j = q - (q / bw) * bw;
+                float f = phi_bias;
+                for (int kh = 0; kh < g.KH; ++kh) {
+                    const int yy = fy0 + i * g.stride + kh;
+                    if (yy < 0 || yy >= g.H) continue;
+                    for (int kw = 0; kw < g.KW; ++kw) {
+                        const int xx = fx0 + j * g.stride + kw;
+                        if (xx < 0 || xx >= g.W) continue;
+                        f += __ldcg(Tn + ((size_t)yy * g.W + xx) * taps + kh * g.KW + kw);
+                    }
+                }
+                best = fmaxf(best, f);
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+            open = best > thr ? 1 : 0;
+        }
+        if (lane == 0) mask[blk] = (uint8_t)open;
+    }
+    if (lane == 0) flags[wid] = open;
+    __syncthreads();
+    if (wid == 0) {
+        const int f = lane < 8 ? flags[lane] : 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, f);
+        int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(count_cur, __popc(bal));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (f) list[base + __popc(bal & ((1u << lane) - 1u))] = (int32_t)(blockIdx.x * 8 + lane);
+    }
+}
+
 GateGeom geom_of(const Layer& L)
 {
     GateGeom g;
@@ -381,6 +501,46 @@ int gate_max_channels(int dtype, bool vec)
 {
     const int es = dtype == SKIPCONV_BF16 ? 2 : 4;
     return vec ? (32 * 4 * 16) / es : 32 * 32;
+}
+
+size_t gumbel_smem_bytes(const Layer& L) { return (size_t)L.p.k_h * L.p.k_w * L.p.c_in * sizeof(float); }
+
+cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
+                                      const uint8_t* chg_prev, uint8_t* chg_cur)
+{
+    const long long n_pix = (long long)L.p.n_streams * L.p.h * L.p.w;
+    const long long blocks = (n_pix + 7) / 8;
+    const long long cap = (long long)L.num_sms * 8;
+    const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
+    const size_t smem = gumbel_smem_bytes(L);
+    const int taps = L.p.k_h * L.p.k_w;
+    if (L.p.dtype == SKIPCONV_BF16)
+        gate_pixel_gumbel_kernel<__nv_bfloat16><<<grid, 256, smem, L.stream>>>(
+            (const __nv_bfloat16*)x_t, (const __nv_bfloat16*)x_prev, (__nv_bfloat16*)x_next, chg_prev, chg_cur,
+            L.gphi, L.pix_taps, n_pix, L.p.c_in, taps, step_count(L), next_count(L));
+    else
+        gate_pixel_gumbel_kernel<float><<<grid, 256, smem, L.stream>>>(
+            (const float*)x_t, (const float*)x_prev, (float*)x_next, chg_prev, chg_cur, L.gphi, L.pix_taps, n_pix,
+            L.p.c_in, taps, step_count(L), next_count(L));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gate_blocks_gumbel(const Layer& L, int force)
+{
+    const GateGeom g = geom_of(L);
+    const long long nblocks = (long long)L.p.n_streams * L.nby * L.nbx;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((nblocks + 7) / 8));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = L.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gate_block_gumbel_kernel, (const float*)L.pix_taps, L.mask, L.list,
+                              step_count(L), g, L.gate_thr, L.gphi_bias, force);
 }
 
 cudaError_t launch_gate_pixels(const Layer& L, const void* x_t, const void* x_prev, void* x_next,

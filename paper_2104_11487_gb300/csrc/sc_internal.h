@@ -29,6 +29,10 @@ struct Layer {
     void* xbuf[2];          // ping-pong x_{t-1} / x_{t-2} frames, dtype
     uint8_t* chg[2];        // per input pixel: x_t != x_{t-1}, for the last two steps
     float* pix_l1;          // per input pixel: sum over channels of |r| (scratch)
+    float* pix_taps;        // Gumbel gate: per input pixel and tap, sum_c phi[tap][c] r[c] (scratch)
+    float* gphi;            // Gumbel gate function phi, [k_h*k_w][c_in] float32
+    float gphi_bias;
+    int gphi_set;           // 1 once skipconv_set_gate_weights was called
     uint8_t* mask;          // [n][nby][nbx]
     int32_t* list;          // active block ids
     int32_t* counters;      // [0], [1]: active-block count of even / odd steps
@@ -86,6 +90,11 @@ inline int32_t* next_count(const Layer& L) { return L.counters + ((L.t + 1) & 1)
 cudaError_t launch_gate_pixels(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
                                const uint8_t* chg_prev, uint8_t* chg_cur, int force);
 cudaError_t launch_gate_blocks(const Layer& L, int force);
+// The Gumbel gate's two passes (Eq. 8): per-pixel tap products, then per-block f and threshold
+size_t gumbel_smem_bytes(const Layer& L);
+cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
+                                      const uint8_t* chg_prev, uint8_t* chg_cur);
+cudaError_t launch_gate_blocks_gumbel(const Layer& L, int force);
 
 // CUDA-core convolution and elementwise kernels (sc_conv_cc.cu)
 cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);

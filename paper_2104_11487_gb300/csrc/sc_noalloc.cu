@@ -191,8 +191,8 @@ extern "C" SKIPCONV_API int skipconv_gate_noalloc(const skipconv_params* params,
     const skipconv_params& p = *params;
     if (!x_t || !x_prev || !block_mask || !active_list || !active_count)
         return set_error("skipconv_gate_noalloc: NULL pointer argument"), SKIPCONV_ERR_INVALID;
-    if (p.gate == SKIPCONV_GATE_OUTPUT)
-        return set_error("skipconv_gate_noalloc: the output-norm gate needs ||w||_1; use a layer handle"),
+    if (p.gate == SKIPCONV_GATE_OUTPUT || p.gate == SKIPCONV_GATE_GUMBEL)
+        return set_error("skipconv_gate_noalloc: the output-norm and Gumbel gates need weights; use a layer handle"),
                SKIPCONV_ERR_UNSUPPORTED;
     const long long n_pix = (long long)p.n_streams * p.h * p.w;
     if (n_pix > SKIPCONV_NOALLOC_MAX_PIXELS)

@@ -595,6 +595,7 @@ cudaError_t prepare_ks(const Layer& L)
 bool step_fused_supported(const Layer& L)
 {
     if (!conv_ws_supported(L) || L.p.dtype != SKIPCONV_BF16 || L.p.stride != 1 || L.p.block != 8) return false;
+    if (L.p.gate == SKIPCONV_GATE_GUMBEL) return false;   // the fused gate warps compute norms only
     const int pb = L.p.c_in * 2;
     // one 16-byte unit per gate lane, 8 to 32 lanes per pixel
     if (pb % 16 != 0 || pb / 16 > 32 || pb / 16 < 5) return false;

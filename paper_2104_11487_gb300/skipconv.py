@@ -10,7 +10,7 @@ from __future__ import annotations
 import ctypes
 
 from . import _lib
-from ._lib import (ACT_NONE, ACT_RELU, ACT_SILU, BF16, F32, GATE_INPUT_MEAN, GATE_INPUT_SUM,  # noqa: F401
+from ._lib import (ACT_NONE, ACT_RELU, ACT_SILU, BF16, F32, GATE_GUMBEL, GATE_INPUT_MEAN, GATE_INPUT_SUM,  # noqa: F401
                    GATE_OUTPUT, PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE, PATH_TENSOR_CORE_SEPARATE, Info,
                    Params, SkipConvError, check)
 
@@ -79,6 +79,10 @@ def skipconv_gate_noalloc(params: Params, x_t, x_prev, block_mask, active_list, 
         _ptr(stream) if stream is not None and not isinstance(stream, int) else stream))
 
 
+def skipconv_set_gate_weights(handle: int, phi_oihw, phi_bias: float = 0.0) -> None:
+    check("skipconv_set_gate_weights", _lib.lib().skipconv_set_gate_weights(handle, _ptr(phi_oihw), float(phi_bias)))
+
+
 def skipconv_get_info(handle: int) -> Info:
     info = Info()
     check("skipconv_get_info", _lib.lib().skipconv_get_info(handle, ctypes.byref(info)))
@@ -119,7 +123,8 @@ class SkipConvLayer:
 
     def __init__(self, n_streams, c_in, c_out, h, w, k=3, stride=1, pad=1, groups=1, block=8, eps=0.05,
                  gate=GATE_INPUT_MEAN, dtype="bf16", activation=ACT_NONE, emit_y=False, dense_mode=False,
-                 conv_path=PATH_AUTO, weights=None, bias=None, stream=None, key_interval=0):
+                 conv_path=PATH_AUTO, weights=None, bias=None, stream=None, key_interval=0, gate_weights=None,
+                 gate_bias=0.0):
         import torch
         self.torch = torch
         self.dtype = torch.bfloat16 if dtype == "bf16" else torch.float32
@@ -131,6 +136,9 @@ class SkipConvLayer:
         b_t = None if bias is None else torch.as_tensor(bias).to(device=dev, dtype=torch.float32).contiguous()
         self.stream = stream if stream is not None else torch.cuda.current_stream(dev)
         self.handle = skipconv_create(self.params, w_t, b_t, self.stream.cuda_stream)
+        if gate_weights is not None:        # Gumbel gate function phi [1, c_in, k, k] (or [c_in, k, k])
+            phi = torch.as_tensor(gate_weights).to(device=dev, dtype=torch.float32).contiguous()
+            skipconv_set_gate_weights(self.handle, phi, gate_bias)
         self.info = skipconv_get_info(self.handle)
         self.shape_in = (n_streams, h, w, c_in)
         self.shape_out = (n_streams, self.info.ho, self.info.wo, c_out)

@@ -40,8 +40,9 @@ def block_max(score: np.ndarray, b: int) -> np.ndarray:
 class Compare:
     """Accumulates per-frame comparison results of one layer."""
 
-    def __init__(self, spec, dtype: str, name: str = ""):
+    def __init__(self, spec, dtype: str, name: str = "", abs_band: float = 0.0):
         self.spec, self.dtype, self.name = spec, dtype, name
+        self.abs_band = abs_band      # absolute exclusion band (threshold 0: the Gumbel gate)
         self.excluded = np.zeros((spec.n, spec.nby, spec.nbx), bool)
         self.max_err = 0.0
         self.max_rel = 0.0
@@ -52,7 +53,7 @@ class Compare:
         s = self.spec
         if not forced:
             bmax = block_max(score, s.block)
-            band = np.abs(bmax - s.eps) <= EPS_BAND * max(s.eps, 1e-30)
+            band = np.abs(bmax - s.eps) <= max(EPS_BAND * max(s.eps, 1e-30), self.abs_band)
             self.n_excluded_events += int(band.sum())
             self.excluded |= band
         else:
@@ -79,7 +80,8 @@ class Compare:
         self.frames += 1
 
 
-def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_path=0, gate=None, key_interval=0):
+def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_path=0, gate=None, key_interval=0,
+              phi=None, phi_bias=0.0):
     import torch
     from paper_2104_11487_gb300 import SkipConvLayer
     wt = torch.from_numpy(np.ascontiguousarray(w, np.float32))
@@ -87,11 +89,14 @@ def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_
     return SkipConvLayer(spec.n, spec.c_in, spec.c_out, spec.h, spec.w, k=spec.k, stride=spec.stride, pad=spec.pad,
                          groups=spec.groups, block=spec.block, eps=spec.eps,
                          gate=spec.gate if gate is None else gate, dtype=dtype, activation=act, emit_y=emit_y,
-                         dense_mode=dense_mode, conv_path=conv_path, weights=wt, bias=bt, key_interval=key_interval)
+                         dense_mode=dense_mode, conv_path=conv_path, weights=wt, bias=bt, key_interval=key_interval,
+                         gate_weights=None if phi is None else torch.from_numpy(np.ascontiguousarray(phi, np.float32)),
+                         gate_bias=phi_bias)
 
 
 def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
-                     reset_at=(), emit_y=False, expect_fused=None, key_interval=0, ref_reset_at=()):
+                     reset_at=(), emit_y=False, expect_fused=None, key_interval=0, ref_reset_at=(), phi=None,
+                     phi_bias=0.0):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record and the conv path used.
     expect_fused: None, or whether the layer must run as one fused launch.
@@ -99,10 +104,10 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
     before which only the oracle is reset (the GPU layer resets itself through
     key_interval)."""
     import oracle
-    ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode)
+    ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode, phi=phi, phi_bias=phi_bias)
     gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y,
-                   key_interval=key_interval)
-    cmp = Compare(spec, dtype, name)
+                   key_interval=key_interval, phi=phi, phi_bias=phi_bias)
+    cmp = Compare(spec, dtype, name, abs_band=1e-4 if spec.gate == oracle.GATE_GUMBEL else 0.0)
     try:
         if expect_fused is not None:
             assert gl.info.fused == int(expect_fused), "%s: fused=%d" % (name, gl.info.fused)

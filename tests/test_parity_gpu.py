@@ -129,6 +129,48 @@ def test_key_interval_resets_like_the_oracle(path):
     assert cmp.frames == 8
 
 
+GUMBEL_CASES = [
+    # name, n, h, w, c_in, c_out, stride, block, dtype
+    ("bf16_b8", 1, 48, 40, 64, 64, 1, 8, "bf16"),
+    ("f32_b1", 1, 32, 24, 32, 32, 1, 1, "f32"),
+    ("f32_stride2_ragged", 2, 37, 29, 16, 24, 2, 4, "f32"),
+]
+
+
+@pytest.mark.parametrize("case", GUMBEL_CASES, ids=[c[0] for c in GUMBEL_CASES])
+@pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
+def test_gumbel_gate(case, path):
+    """Gumbel gate at inference (Eq. 8): f(r; phi) > 0 with a random one-output-
+    channel phi and a negative bias, so that small residuals stay closed."""
+    from oracle import GATE_GUMBEL
+    name, n, h, w, c_in, c_out, stride, block, dtype = case
+    if path == AUTO and stride != 1 and dtype == "bf16":
+        pytest.skip("covered by the CUDA-core case")
+    rng = np.random.default_rng(400 + block)
+    v = np.stack([synth.moving_squares_video(41 + s, 5, h, w, c_in, n_squares=2, size=8, speed=3, noise_std=0.01)
+                  for s in range(n)], axis=1)
+    frames = synth.round_to_bf16(v) if dtype == "bf16" else v.astype(np.float32)
+    wts = synth.he_weights(rng, c_out, c_in, 3, bf16=dtype == "bf16")
+    phi = (rng.standard_normal((c_in, 3, 3)) * 0.2).astype(np.float32)
+    spec = LayerSpec(n=n, c_in=c_in, c_out=c_out, h=h, w=w, k=3, stride=stride, pad=1, block=block, eps=0.0,
+                     gate=GATE_GUMBEL)
+    cmp, _ = run_single_layer(spec, wts, None, [frames[t] for t in range(5)], dtype, conv_path=path,
+                              name="gumbel " + name, phi=phi, phi_bias=-0.3, expect_fused=False)
+    assert cmp.frames == 5
+
+
+def test_gumbel_gate_needs_weights():
+    import torch
+    from paper_2104_11487_gb300 import SkipConvLayer, skipconv_step
+    from paper_2104_11487_gb300._lib import SkipConvError, SKIPCONV_ERR_INVALID
+    w = torch.zeros((8, 8, 3, 3))
+    lay = SkipConvLayer(1, 8, 8, 16, 16, block=8, eps=0.0, gate=3, dtype="f32", weights=w)
+    with pytest.raises(SkipConvError) as ei:
+        skipconv_step(lay.handle, torch.zeros((1, 16, 16, 8), device="cuda"))
+    assert ei.value.status == SKIPCONV_ERR_INVALID and "skipconv_set_gate_weights" in str(ei.value)
+    lay.close()
+
+
 def test_zero_residual_keeps_state_bitwise():
     import torch
     from harness import gpu_layer
