@@ -339,6 +339,53 @@ def cpu_oracle_sample(seconds, density, max_frames=40):
                       "double-precision C loops" % (done, t_total)}
 
 
+# ------------------------------------------------------------- ranks
+class Ranks:
+    """Process-group plumbing of a replica run (torchrun, one rank per GPU):
+    every rank runs its own streams, there is no collective on the data path;
+    ranks meet only at barriers around the timed region and to take the
+    slowest rank's time.  backend/device: "nccl"/"cuda" on GPUs, "gloo"/"cpu"
+    in the CPU tests."""
+
+    def __init__(self, backend="nccl", device="cuda"):
+        import torch
+        self.torch = torch
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.device = device
+        self.dist = None
+        if self.world > 1:
+            import torch.distributed as dist
+            kw = {"device_id": torch.device("cuda", self.local)} if device == "cuda" else {}
+            dist.init_process_group(backend, **kw)
+            self.dist = dist
+
+    def barrier(self):
+        if self.dist:
+            self.dist.barrier()
+        if self.device == "cuda":
+            self.torch.cuda.synchronize()
+
+    def max(self, v: float) -> float:
+        """The largest v over all ranks (the slowest rank's time)."""
+        if not self.dist:
+            return v
+        t = self.torch.tensor([v], dtype=self.torch.float64, device=self.device)
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.dist:
+            self.dist.destroy_process_group()
+
+
+def replica_value(world: int, steps: int, total_ms: float) -> float:
+    """Whole-job stream-frames/s: the stream-frames of all ranks over the
+    slowest rank's time."""
+    return world * N_STREAMS * steps / (total_ms / 1e3)
+
+
 # ---------------------------------------------------------------- main
 def main():
     args = parse()
@@ -353,22 +400,8 @@ def main():
 
     import torch
     torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    def barrier():
-        if dist:
-            dist.barrier()
-        torch.cuda.synchronize()
-
-    def max_over_ranks(v):
-        if not dist:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    ranks = Ranks()
+    barrier, max_over_ranks = ranks.barrier, ranks.max
 
     from paper_2104_11487_gb300 import _lib, skipconv_get_info
     _lib.lib()
@@ -396,7 +429,7 @@ def main():
     clk["window"] = "every 100 ms over the timed steps and 0.5 s of the same steps before and after"
     total_ms = max_over_ranks(sum(ms))
     ms_per_step = total_ms / args.steps
-    value = world * N_STREAMS * args.steps / (total_ms / 1e3)
+    value = replica_value(world, args.steps, total_ms)
 
     # 2) the same steps with per-kernel CUDA events (dominant kernel's roofline)
     ms_p, launches_p, kms, counts, _ = run_layer_timed(layer, frames, args.warmup, args.steps, flush, torch,
@@ -464,7 +497,7 @@ def main():
         for i in range(args.steps):
             skipconv_step_host(layer.handle, host[args.warmup + 1 + i], zh)
         t_e2e = max_over_ranks(time.perf_counter() - t0)
-        line["e2e"] = {"value": world * N_STREAMS * args.steps / t_e2e, "unit": UNIT,
+        line["e2e"] = {"value": replica_value(world, args.steps, t_e2e * 1e3), "unit": UNIT,
                        "h2d_bytes_per_step": host[0].numel() * 2, "d2h_bytes_per_step": zh.numel() * 4,
                        "call": "skipconv_step_host (synchronous; host frame in, full fp32 z out)"}
         del host
@@ -505,8 +538,7 @@ def main():
         line["drift_vs_dense"] = drift_report(torch)
     if rank == 0:
         print(json.dumps(line), flush=True)
-    if dist:
-        dist.destroy_process_group()
+    ranks.close()
     return 0
 
 
