@@ -34,7 +34,7 @@ METRIC = "Skip-Conv frames/s and effective TFLOP/s vs roofline at measured gate 
 UNIT = "stream-frames/s"
 N_STREAMS, H, W, C, K, BLOCK, EPS = 8, 128, 128, 256, 3, 8, 0.05
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KERNELS = ("gate_pixel", "gate_block", "conv", "y_refresh", "step_fused")
+KERNELS = ("gate_pixel", "gate_block", "conv", "y_refresh", "step_fused", "step_local")
 
 
 def parse():
@@ -56,6 +56,8 @@ def parse():
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the single-layer and stacked workloads (c0-c3)")
     ap.add_argument("--no-flush", action="store_true",
                     help="no L2 flush between timed steps: each step streams 134 MB of frames, more than the L2")
     ap.add_argument("--no-soak", action="store_true",
@@ -311,6 +313,145 @@ def drift_report(torch, intervals=(0, 4, 8, 16), T=32):
             "reference": "the same layer reset at every step (z_t = w * x_t + b)", "key_interval": out}
 
 
+# -------------------------------------------------- the other workloads
+ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12      # fp32 FMA: SMs x FMA lanes x 2 FLOP x max SM clock
+
+
+def layer_roof(L, n, h, w, ho, wo, esz, locs, chg, emit_y, conv_path, tc_peak, hbm):
+    """Algorithmic FLOPs and bytes of one layer step and its roofline time:
+    full reads of x_t and x_{t-1}, the commit of changed pixels, the fp32 z
+    read-modify-write at the open locations, the weights, and y: written at
+    the open locations, or (with a shortcut) refreshed over the whole frame
+    from z and the shortcut.  Dense layers on the tensor path use the bf16
+    tensor peak; CUDA-core layers (fp32, depthwise) the fp32 FMA peak."""
+    flops = 2.0 * locs * L.c_out * (L.c_in // L.groups) * L.k * L.k
+    x = n * h * w * L.c_in * esz
+    bytes_ = 2 * x + chg * L.c_in * esz + 2 * locs * L.c_out * 4 + L.c_out * (L.c_in // L.groups) * L.k * L.k * esz
+    if L.shortcut >= 0:
+        bytes_ += n * ho * wo * L.c_out * (4 + 2 * esz)
+    elif emit_y:
+        bytes_ += locs * L.c_out * esz
+    peak = tc_peak if conv_path == 2 else ALU_TFLOPS
+    return flops, bytes_, max(flops / (peak * 1e12), bytes_ / (hbm * 1e9))
+
+
+def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c2", "c3")):
+    """The single-layer (c0, c1) and stacked (c2 pose-like, c3 MBConv-like)
+    workloads, run free: each layer steps on the previous layer's y (and its
+    shortcut) on the device, one frame after the other, with an L2 flush
+    between frames.  Frame 0 is the key frame; `warmup` frames follow
+    untimed; the rest of the video is timed with CUDA events around each
+    frame.  A second pass with the library's per-launch events gives each
+    layer's kernel time, and a third (host-synchronised) pass counts each
+    layer's open locations and changed input pixels for its roofline."""
+    import synth
+    from paper_2104_11487_gb300 import (SkipConvLayer, device_tensor, skipconv_get_y, skipconv_profile,
+                                        skipconv_profile_read)
+    report = {}
+    for name in names:
+        wl = synth.make_workload(name)
+        dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+        esz = 2 if wl.dtype == "bf16" else 4
+        frames = [torch.from_numpy(np.ascontiguousarray(wl.frames[t])).cuda().to(dt) for t in range(wl.T)]
+        stacked = len(wl.layers) > 1
+        lays, ys, dims = [], [], []
+        h, w = wl.h, wl.w
+        for li, L in enumerate(wl.layers):
+            lay = SkipConvLayer(wl.n, L.c_in, L.c_out, h, w, k=L.k, stride=L.stride, pad=L.pad, groups=L.groups,
+                                block=L.block, eps=L.eps, dtype=wl.dtype, activation=L.act, emit_y=stacked,
+                                weights=torch.from_numpy(wl.weights[li]),
+                                bias=None if wl.biases[li] is None else torch.from_numpy(wl.biases[li]))
+            lays.append(lay)
+            ys.append(device_tensor(skipconv_get_y(lay.handle), lay.shape_out, dt) if stacked else None)
+            dims.append((h, w, lay.info.ho, lay.info.wo))
+            h, w = lay.info.ho, lay.info.wo
+        stream = lays[0].stream
+
+        def frame_step(x):
+            stack = [x]
+            for li, L in enumerate(wl.layers):
+                lays[li].step(stack[-1], None if L.shortcut < 0 else stack[L.shortcut])
+                stack.append(ys[li])
+
+        def reset():
+            for lay in lays:
+                lay.reset()
+
+        timed = range(warmup + 1, wl.T)
+        # 1) whole frames
+        reset()
+        for t in range(warmup + 1):
+            frame_step(frames[t])
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in timed]
+        torch.cuda.synchronize()
+        for i, t in enumerate(timed):
+            flush_l2(flush)
+            ev[i][0].record(stream)
+            frame_step(frames[t])
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        ms = [a.elapsed_time(b) for a, b in ev]
+        # 2) per-layer kernel time (library events around each launch)
+        reset()
+        for t in range(warmup + 1):
+            frame_step(frames[t])
+        for lay in lays:
+            skipconv_profile(lay.handle, True)
+        for t in timed:
+            flush_l2(flush)
+            frame_step(frames[t])
+        torch.cuda.synchronize()
+        layer_ms, layer_launches = [], []
+        for lay in lays:
+            launches, kms = skipconv_profile_read(lay.handle)
+            skipconv_profile(lay.handle, False)
+            layer_ms.append(sum(kms) / len(timed))
+            layer_launches.append(sum(launches) / len(timed))
+        # 3) open locations and changed input pixels per layer (untimed, synchronised)
+        reset()
+        locs = [[] for _ in lays]
+        chg = [[] for _ in lays]
+        prev_in = [None] * len(lays)
+        for t in range(wl.T):
+            stack = [frames[t]]
+            for li, L in enumerate(wl.layers):
+                x = stack[-1]
+                if t in timed:
+                    chg[li].append(int((x != prev_in[li]).any(dim=-1).sum()))
+                    lays[li].step(x, None if L.shortcut < 0 else stack[L.shortcut])
+                    locs[li].append(lays[li].stats()[1])
+                else:
+                    lays[li].step(x, None if L.shortcut < 0 else stack[L.shortcut])
+                prev_in[li] = x.clone()
+                stack.append(ys[li])
+        per_layer, t_roof_sum, flops_sum = [], 0.0, 0.0
+        for li, L in enumerate(wl.layers):
+            h_, w_, ho, wo = dims[li]
+            loc = statistics.mean(locs[li])
+            fl, by, tr = layer_roof(L, wl.n, h_, w_, ho, wo, esz, loc, statistics.mean(chg[li]), stacked,
+                                    lays[li].info.conv_path, tc_peak, hbm)
+            t_roof_sum += tr
+            flops_sum += fl
+            per_layer.append({"layer": L.name, "shape": "%dx%dx%d -> %dx%dx%d, k%d s%d g%d, b%d" % (
+                h_, w_, L.c_in, ho, wo, L.c_out, L.k, L.stride, L.groups, L.block),
+                "path": {1: "cuda-core", 2: "tensor-core"}.get(lays[li].info.conv_path),
+                "fused": bool(lays[li].info.fused), "launches": layer_launches[li],
+                "open_location_density": loc / (wl.n * ho * wo), "kernel_us": layer_ms[li] * 1e3,
+                "eff_tflops": fl / (layer_ms[li] * 1e-3) / 1e12 if layer_ms[li] else None,
+                "roofline_frac": tr / (layer_ms[li] * 1e-3) if layer_ms[li] else None})
+        t_frame = statistics.median(ms) * 1e-3
+        report[name] = {"frames": len(timed), "dtype": wl.dtype, "ms_per_frame": t_frame * 1e3,
+                        "frames_per_s": wl.n / t_frame, "eff_tflops": flops_sum / t_frame / 1e12,
+                        "stack_roofline_frac": t_roof_sum / t_frame, "layers": per_layer}
+        for lay in lays:
+            lay.close()
+        del frames
+    return {"note": "frames/s and the stack roofline fraction use the median frame time (CUDA events, L2 flushed "
+                    "between frames); each layer's fraction uses its kernels' event time; CUDA-core layers are "
+                    "measured against %.1f TFLOP/s fp32 FMA (152 SMs x 128 lanes x 2 x 2.07 GHz)" % ALU_TFLOPS,
+            "workloads": report}
+
+
 # ----------------------------------------------------------- CPU oracle
 def cpu_oracle_sample(seconds, density, max_frames=40):
     """The oracle as it stands, on the host cores: stream 0 of the same
@@ -530,7 +671,11 @@ def main():
             s["faster_than_dense_mode"] = (s["ms_per_step"] < dense_ms) if dense_ms else None
         line["sweep"] = {"points": sweep, "dense_mode_ms_per_step": dense_ms}
 
-    # 5) the CPU oracle on the host cores (rank 0, N = 1 only)
+    # 5) the single-layer and stacked workloads
+    if not args.no_workloads:
+        line["other_workloads"] = workloads_report(torch, flush, tc_peak, hbm)
+
+    # 6) the CPU oracle on the host cores (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_oracle_sample(args.cpu_seconds, args.density)
     layer.close()

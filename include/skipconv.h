@@ -80,11 +80,17 @@ typedef enum { SKIPCONV_F32 = 0, SKIPCONV_BF16 = 1 } skipconv_dtype;
 typedef enum { SKIPCONV_ACT_NONE = 0, SKIPCONV_ACT_RELU = 1, SKIPCONV_ACT_SILU = 2 } skipconv_act;
 
 typedef enum {
-    SKIPCONV_PATH_AUTO = 0,        /* tensor cores where supported, else CUDA cores */
+    SKIPCONV_PATH_AUTO = 0,        /* tensor cores where supported, else CUDA cores;
+                                      layers whose dense step is at most 2^26 MACs
+                                      run the one-launch CUDA-core step (a step of
+                                      that size is latency-bound)                 */
     SKIPCONV_PATH_CUDA_CORE = 1,   /* float32 FMA direct convolution              */
     SKIPCONV_PATH_TENSOR_CORE = 2, /* tcgen05 implicit GEMM (bf16 in, fp32 accum)  */
-    SKIPCONV_PATH_TENSOR_CORE_SEPARATE = 3 /* the same convolution, but never fused with
+    SKIPCONV_PATH_TENSOR_CORE_SEPARATE = 3, /* the same convolution, but never fused with
                                       the gate: three launches per step           */
+    SKIPCONV_PATH_CUDA_CORE_SEPARATE = 4 /* the CUDA-core convolution in its own launch
+                                      after the two gate passes (CUDA_CORE runs the
+                                      whole step as one launch where it can)      */
 } skipconv_path;
 
 typedef struct {
@@ -169,8 +175,11 @@ typedef struct {
     int conv_path;     /* path actually used: SKIPCONV_PATH_CUDA_CORE or _TENSOR_CORE */
     int num_sms;       /* SMs of the device the handle lives on               */
     size_t state_bytes;/* device bytes held by the handle                     */
-    int fused;         /* 1: each step is one fused launch (gate and convolution
-                          pipelined over the streams), 0: separate launches  */
+    int fused;         /* 0: separate launches (gate passes, convolution, y);
+                          1: each step is one cooperative tensor-core launch
+                          (gate and convolution pipelined over the streams);
+                          2: each step is one CUDA-core launch, a CTA per tile
+                          of gate blocks working from its own input footprint */
 } skipconv_info;
 SKIPCONV_API int skipconv_get_info(skipconv_handle h, skipconv_info* info);
 
@@ -187,11 +196,12 @@ SKIPCONV_API int skipconv_check_device(skipconv_handle h);
 
 /* Per-kernel timing.  Kernel kinds: 0 gate_pixel (residual, channel l1 norm,
  * state commit), 1 gate_block (support norm, block gate, compaction), 2 the
- * convolution of the open blocks (either path), 3 y refresh, 4 the fused step
- * (all of 0-2 in one launch).  Launch counts are always kept; with enable = 1
+ * convolution of the open blocks (either path), 3 y refresh, 4 the fused
+ * tensor-core step (all of 0-2 in one launch), 5 the one-launch CUDA-core step
+ * (all of 0-3).  Launch counts are always kept; with enable = 1
  * each launch is also bracketed by CUDA events on the handle's stream.
  * skipconv_profile resets both. */
-#define SKIPCONV_PROFILE_KINDS 5
+#define SKIPCONV_PROFILE_KINDS 6
 SKIPCONV_API int skipconv_profile(skipconv_handle h, int enable);
 /* Synchronise the stream and report, per kernel kind (arrays of
  * SKIPCONV_PROFILE_KINDS), the launches and the summed event-timed

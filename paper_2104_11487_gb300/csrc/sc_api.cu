@@ -1,6 +1,7 @@
 // Host side of the Skip-Conv C ABI (include/skipconv.h): argument checks,
 // state allocation, weight repacking, and the per-step launch sequence
-//   step_fused (one launch), or
+//   step_fused (one cooperative tensor-core launch), or
+//   step_local (one CUDA-core launch, a CTA per tile of gate blocks), or
 //   gate_pixel -> gate_block -> conv (tensor-core or CUDA-core) [-> y_refresh]
 // all on the handle's stream, with no host synchronisation per step.
 #include <stdarg.h>
@@ -8,6 +9,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -25,6 +27,21 @@ void set_error(const char* fmt, ...)
     va_start(ap, fmt);
     vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
     va_end(ap);
+}
+
+// cudaFuncAttributeMaxDynamicSharedMemorySize belongs to the kernel, not to a
+// layer: layers that share a kernel but need different amounts must only ever
+// raise it, or the last layer created would lower it below what an earlier
+// one launches with.
+cudaError_t ensure_dynamic_smem(const void* func, size_t bytes)
+{
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, func);
+    if (e != cudaSuccess) return e;
+    if ((size_t)fa.maxDynamicSharedSizeBytes >= bytes) return cudaSuccess;
+    return cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
 EncodeTiledFn encode_tiled_fn()
@@ -122,7 +139,7 @@ static void free_buffers(Layer* L)
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
                     L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag,
-                    L->pix_taps, L->gphi};
+                    L->pix_taps, L->gphi, L->w_loc};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);
@@ -162,7 +179,7 @@ int validate(const skipconv_params* p)
         return set_error("unknown dtype %d", p->dtype), SKIPCONV_ERR_INVALID;
     if (p->activation < SKIPCONV_ACT_NONE || p->activation > SKIPCONV_ACT_SILU)
         return set_error("unknown activation %d", p->activation), SKIPCONV_ERR_INVALID;
-    if (p->conv_path < SKIPCONV_PATH_AUTO || p->conv_path > SKIPCONV_PATH_TENSOR_CORE_SEPARATE)
+    if (p->conv_path < SKIPCONV_PATH_AUTO || p->conv_path > SKIPCONV_PATH_CUDA_CORE_SEPARATE)
         return set_error("unknown conv_path %d", p->conv_path), SKIPCONV_ERR_INVALID;
     const long long frame = (long long)p->n_streams * p->h * p->w;
     if (frame * p->c_in > (1LL << 40)) return set_error("frame too large"), SKIPCONV_ERR_INVALID;
@@ -247,13 +264,11 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         delete h;
         return SKIPCONV_ERR_UNSUPPORTED;
     }
-    L.path = (L.p.conv_path == SKIPCONV_PATH_CUDA_CORE || !tc_ok) ? SKIPCONV_PATH_CUDA_CORE
-                                                                   : SKIPCONV_PATH_TENSOR_CORE;
-    if (L.path == SKIPCONV_PATH_CUDA_CORE && conv_cc_smem_bytes(L) > 200 * 1024) {
-        set_error("CUDA-core path: halo tile of %zu bytes exceeds shared memory", conv_cc_smem_bytes(L));
-        delete h;
-        return SKIPCONV_ERR_UNSUPPORTED;
-    }
+    const bool want_cc = L.p.conv_path == SKIPCONV_PATH_CUDA_CORE ||
+                         L.p.conv_path == SKIPCONV_PATH_CUDA_CORE_SEPARATE;
+    // AUTO: small layers (latency-bound steps) take the one-launch CUDA-core step
+    const bool small = L.p.conv_path == SKIPCONV_PATH_AUTO && step_local_preferred(L);
+    L.path = (want_cc || small || !tc_ok) ? SKIPCONV_PATH_CUDA_CORE : SKIPCONV_PATH_TENSOR_CORE;
     L.ci_pad = ((L.p.c_in + 63) / 64) * 64;
     L.co_pad = ((L.p.c_out + 127) / 128) * 128;
 
@@ -354,6 +369,11 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         }
         L.state_bytes = A.bytes;
     }
+    // CUDA-core layers: the whole step as one launch, unless the separate launches were asked for
+    if (e == cudaSuccess && step_local_supported(L)) {
+        e = step_local_prepare(L);
+        if (e == cudaSuccess) L.fused = 2;
+    }
     if (e == cudaSuccess) {
         h->L.key = 1;
         st = skipconv_reset_state(h);
@@ -411,8 +431,10 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     // chg[nxt] marks pixels that changed at the previous step; chg[cur] is written now.
     const int force = (L->key || L->p.dense_mode) ? 1 : 0;
     if (L->fused) {
-        const int slot = prof_begin(L, 4);
-        const cudaError_t e = launch_step_fused(*L, x_t, force);
+        const int kind = L->fused == 1 ? 4 : 5;
+        const int slot = prof_begin(L, kind);
+        const cudaError_t e = L->fused == 1 ? launch_step_fused(*L, x_t, force)
+                                            : launch_step_local(*L, x_t, shortcut, force);
         prof_end(L, slot);
         if (e != cudaSuccess) return status_of(e);
         L->since_key = force && L->key ? 1 : L->since_key + 1;

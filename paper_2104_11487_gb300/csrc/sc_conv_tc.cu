@@ -411,8 +411,7 @@ cudaError_t conv_tc_prepare(Layer& L)
     }
     L.tc_z_tma = tc_encode_z_map(&L.tmap_z, L) ? 1 : 0;
     const int HH = 8 + L.p.k_h - 1, WW = 8 + L.p.k_w - 1;
-    return cudaFuncSetAttribute(conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)tc_smem_bytes(HH, WW));
+    return ensure_dynamic_smem((const void*)conv_tc_kernel, tc_smem_bytes(HH, WW));
 }
 
 cudaError_t launch_conv_tc(const Layer& L, const void* x_t, const void* x_prev, int prev_index)

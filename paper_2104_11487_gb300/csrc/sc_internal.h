@@ -39,7 +39,7 @@ struct Layer {
     float* z;               // [n][ho][wo][c_out]
     void* y;                // [n][ho][wo][c_out] dtype or NULL
     float* bias;            // [c_out]
-    float* w_cc;            // [cpg][k_h][k_w][c_out] fp32 (CUDA-core path)
+    float* w_cc;            // [k_h][k_w][cpg][c_out] fp32 (CUDA-core path)
     __nv_bfloat16* w_tc;    // [co_pad][k_h*k_w*ci_pad] bf16 (tensor-core path)
     int ci_pad, co_pad;     // tensor-core padding of c_in (multiple of 64) and c_out (of 128)
     void* x_stage;          // device staging frame for skipconv_step_host (lazy)
@@ -72,11 +72,16 @@ struct Layer {
     CUtensorMap tmap_z;
 
     // fused step kernel (sc_step_fused.cu)
-    int fused;              // 1: the whole step is one cooperative launch
+    int fused;              // 1: the step is one cooperative tensor-core launch; 2: one CUDA-core launch
     int* sched;             // fused step: grid abort flag (16 ints reserved)
     uint64_t* pnorm;        // fused step: per pixel (epoch << 32) | fp32 norm
     uint32_t* gtag;         // fused step: per gate block (epoch << 1) | open
     uint32_t epoch;         // fused step: tag of the last launched step
+
+    // one-launch CUDA-core step (sc_step_local.cu)
+    int local_staged;       // 1: its TMA-footprint / staged-weight form
+    CUtensorMap tmap_fp[2]; // footprint boxes of the two state frames
+    void* w_loc;            // weights packed per CTA slice, layer dtype
 };
 
 // ------------------------------------------------------------------ launchers
@@ -101,7 +106,6 @@ cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
 cudaError_t launch_y_refresh(const Layer& L, const void* shortcut);
 cudaError_t launch_reset_z(const Layer& L);
 cudaError_t launch_pack_weights(Layer& L, const void* w_oihw, double* w_l1_out);
-size_t conv_cc_smem_bytes(const Layer& L);
 
 // Tensor-core convolution (sc_conv_tc.cu)
 bool conv_tc_supported(const skipconv_params& p, const char** why);
@@ -119,6 +123,19 @@ bool step_fused_supported(const Layer& L);
 cudaError_t step_fused_prepare(Layer& L);
 cudaError_t launch_step_fused(Layer& L, const void* x_t, int force);
 
+// One-launch step for CUDA-core layers (sc_step_local.cu): a CTA per tile of
+// gate blocks computes residual, norms, gates, convolution, y and the commit
+// from its own input footprint.
+constexpr size_t LOCAL_MAX_SMEM = 200 * 1024;
+// Layers whose dense step is at most this many MACs run on this form under
+// SKIPCONV_PATH_AUTO even where tensor cores could serve them: at that size a
+// step is bound by latency (a few memory round trips), not by arithmetic.
+constexpr double LOCAL_AUTO_MAX_MACS = 67108864.0;   // 2^26
+bool step_local_preferred(const Layer& L);
+bool step_local_supported(const Layer& L);
+cudaError_t step_local_prepare(Layer& L);
+cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* shortcut, int force);
+
 // Driver entry point for tensor-map encoding (resolved once through the runtime).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -126,6 +143,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 EncodeTiledFn encode_tiled_fn();
 
 void set_error(const char* fmt, ...);
+// Raise (never lower) a kernel's dynamic shared-memory limit to `bytes`.
+cudaError_t ensure_dynamic_smem(const void* func, size_t bytes);
 // Host-side check of a parameter block (sizes, enums, limits); sets the error text.
 int validate(const skipconv_params* p);
 

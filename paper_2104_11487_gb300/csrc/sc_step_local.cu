@@ -1,0 +1,1011 @@
+// One-launch Skip-Conv step for layers on the CUDA-core path.
+//
+// Every CTA takes a tile of sb x sb gate blocks and does the whole step for
+// it from its own input footprint (the union of the receptive fields of the
+// tile's output locations):
+//   1. r_t = x_t - x_{t-1} over the footprint (Eq. 2), kept in shared memory
+//      as float32, and each pixel's l1 norm over all input channels;
+//   2. the commit of x_t into the ping-pong buffer that becomes x_{t-1} at the
+//      next step, for the input pixels this tile owns (pixels that changed at
+//      this step or the previous one), and the pixels' change flags;
+//   3. the block gates: per output location the norms summed over its
+//      k_h x k_w receptive field (the local support norm of Eq. 5), the block
+//      maximum (max-pooling of the gate, Sec. 3.2) against the threshold;
+//   4. the open blocks appended to the compact list (one atomic per tile);
+//   5. w * r_t at the open locations, added into z in place (Eq. 3), from the
+//      shared-memory residual: a register-blocked contraction over
+//      k_h*k_w*(c_in/groups) on float32 FMAs (dense and grouped layers), or
+//      one thread per channel and location (depthwise);
+//   6. y = act(z) at the open locations, or y = act(z + shortcut) over the
+//      whole tile when the layer has a shortcut.
+// Halo pixels shared with neighbouring tiles are recomputed instead of
+// exchanged, so no CTA waits on another, and the launch is a programmatic
+// dependent of the previous kernel in the stream (typically the layer that
+// produced x_t): its CTAs are scheduled while that kernel drains and start
+// reading x_t once it has completed.
+//
+// Two forms.  The staged form (dense layers with groups = 1, and depthwise
+// layers, when a pixel's channels are a multiple of 16 bytes and at most 256)
+// gives each CTA one slice of SW output channels of a tile (depthwise: all
+// channels) and moves its data with asynchronous copies: the slice's weights
+// with one bulk copy issued before the dependency wait (they are constant
+// state), the x_t and x_{t-1} footprints as two TMA boxes right after it
+// (zero fill outside the frame is the convolution's zero padding), so that a
+// step costs about three memory round trips (footprint, weights in parallel,
+// z).  The contraction is split over k when the open locations are too few
+// to occupy the CTA.  The general form loads with plain per-thread accesses
+// and reads weights from global memory; it serves every other shape.
+#include "sc_internal.h"
+#include "sc_ptx.cuh"
+
+namespace sc {
+namespace {
+
+using namespace ptx;
+
+constexpr int LT = 128;               // threads per CTA
+constexpr int LPI = 2;                // output locations per work item of the dense contraction
+constexpr int MAX_TILE_BLOCKS = 16;   // sb <= 4
+
+struct LocalArgs {
+    const void* xt;
+    const void* xp;            // x_{t-1}
+    void* xn;                  // receives x_t (holds x_{t-2})
+    const uint8_t* chg_prev;   // pixels that changed at the previous step
+    uint8_t* chg_cur;          // pixels that change at this step
+    const float* wcc;          // [k_h][k_w][cpg][c_out] float32
+    float* z;
+    void* y;                   // or NULL
+    const void* sc;            // shortcut, or NULL
+    uint8_t* mask;
+    int32_t* list;
+    int32_t* count_cur;        // this step's open-block count (zeroed by the previous step or the reset)
+    int32_t* count_next;       // zeroed here for the next step
+    int force;                 // key frame or dense mode: every block open
+    int n, H, W, C, Ho, Wo, Co, KH, KW, stride, pad, b, nby, nbx, cpg, opg, groups, act;
+    int sb, nty, ntx, FH, FW, CP;
+    float thr;                 // threshold on the raw local l1 sum
+};
+
+__device__ __forceinline__ unsigned bits_of(float v) { return __float_as_uint(v); }
+__device__ __forceinline__ unsigned bits_of(__nv_bfloat16 v) { return (unsigned)__bfloat16_as_ushort(v); }
+
+__device__ __forceinline__ float warp_sum(float v)
+{
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    return v;
+}
+
+__device__ __forceinline__ float warp_max(float v)
+{
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+    return v;
+}
+
+template <typename T, bool DW, bool V4>
+__global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
+{
+    extern __shared__ __align__(16) float sm[];
+    __shared__ int s_open[MAX_TILE_BLOCKS];
+    __shared__ int s_nloc;
+    const int FP = a.FH * a.FW;
+    float* R = sm;                                   // [FP][CP] residual of the footprint
+    float* P = R + (size_t)FP * a.CP;                // [FP] per-pixel l1 norm
+    int* locs = reinterpret_cast<int*>(P + FP);      // open output locations of the tile, (li << 16) | lj
+
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    const T* xt = static_cast<const T*>(a.xt);
+    const T* xp = static_cast<const T*>(a.xp);
+    T* xn = static_cast<T*>(a.xn);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int NW = LT / 32;
+    const int tile = blockIdx.x;
+    const int tx = tile % a.ntx, ty = (tile / a.ntx) % a.nty, nn = tile / (a.ntx * a.nty);
+    const int span = a.sb * a.b;                     // output locations per tile side
+    const int oy0 = ty * span, ox0 = tx * span;
+    const int fy0 = oy0 * a.stride - a.pad, fx0 = ox0 * a.stride - a.pad;
+    if (tile == 0 && threadIdx.x == 0) *a.count_next = 0;
+    if (threadIdx.x == 0) s_nloc = 0;
+
+    const int own_y0 = min(ty * span * a.stride, a.H);
+    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
+    const int own_x0 = min(tx * span * a.stride, a.W);
+    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
+    const int ow = own_x1 - own_x0, npx = (own_y1 - own_y0) * ow;
+    if (a.C <= 16) {
+        // few channels: a thread per pixel, so that every pixel's loads are in flight at once
+        // 1. residual of the footprint and per-pixel norms
+        for (int q = threadIdx.x; q < FP; q += LT) {
+            const int iy = fy0 + q / a.FW, ix = fx0 + q % a.FW;
+            const bool in = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+            const size_t base = in ? (((size_t)nn * a.H + iy) * a.W + ix) * a.C : 0;
+            float s = 0.f;
+            for (int c = 0; c < a.C; ++c) {
+                const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
+                R[(size_t)q * a.CP + c] = r;
+                s += fabsf(r);
+            }
+            P[q] = s;
+        }
+        // 2. commit x_t for the input pixels this tile owns (each input pixel has exactly one owner)
+        for (int q = threadIdx.x; q < npx; q += LT) {
+            const size_t pix = ((size_t)nn * a.H + own_y0 + q / ow) * a.W + own_x0 + q % ow;
+            const size_t base = pix * a.C;
+            unsigned d = 0;
+            for (int c = 0; c < a.C; ++c) d |= bits_of(xt[base + c]) ^ bits_of(xp[base + c]);
+            if (d || a.chg_prev[pix])
+                for (int c = 0; c < a.C; ++c) xn[base + c] = xt[base + c];
+            a.chg_cur[pix] = d ? 1 : 0;
+        }
+    } else {
+        // 1. residual of the footprint and per-pixel norms (a warp per pixel, lanes over channels)
+        for (int q = warp; q < FP; q += NW) {
+            const int fy = q / a.FW, fx = q - (q / a.FW) * a.FW;
+            const int iy = fy0 + fy, ix = fx0 + fx;
+            const bool in = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+            const size_t base = in ? (((size_t)nn * a.H + iy) * a.W + ix) * a.C : 0;
+            float s = 0.f;
+            for (int c = lane; c < a.C; c += 32) {
+                const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
+                R[(size_t)q * a.CP + c] = r;
+                s += fabsf(r);
+            }
+            s = warp_sum(s);
+            if (lane == 0) P[q] = s;
+        }
+        // 2. commit x_t for the input pixels this tile owns (each input pixel has exactly one owner)
+        for (int q = warp; q < npx; q += NW) {
+            const int iy = own_y0 + q / ow, ix = own_x0 + q % ow;
+            const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
+            const size_t base = pix * a.C;
+            unsigned d = 0;
+            for (int c = lane; c < a.C; c += 32) d |= bits_of(xt[base + c]) ^ bits_of(xp[base + c]);
+            const bool changed = __any_sync(0xffffffffu, d != 0);
+            if (changed || a.chg_prev[pix])
+                for (int c = lane; c < a.C; c += 32) xn[base + c] = xt[base + c];
+            if (lane == 0) a.chg_cur[pix] = changed ? 1 : 0;
+        }
+    }
+    __syncthreads();
+
+    // 3. block gates of the tile (a warp per gate block)
+    for (int bq = warp; bq < a.sb * a.sb; bq += NW) {
+        const int bi = bq / a.sb, bj = bq - (bq / a.sb) * a.sb;
+        const int by = ty * a.sb + bi, bx = tx * a.sb + bj;
+        int open = 0;
+        if (by < a.nby && bx < a.nbx) {
+            const int bh = min(a.b, a.Ho - by * a.b), bw = min(a.b, a.Wo - bx * a.b);
+            float best = -1.f;
+            for (int q = lane; q < bh * bw; q += 32) {
+                const int li = bi * a.b + q / bw, lj = bj * a.b + q % bw;
+                float S = 0.f;
+                for (int kh = 0; kh < a.KH; ++kh)
+                    for (int kw = 0; kw < a.KW; ++kw) S += P[(li * a.stride + kh) * a.FW + lj * a.stride + kw];
+                best = fmaxf(best, S);
+            }
+            best = warp_max(best);
+            open = (a.force || best > a.thr) ? 1 : 0;
+            if (lane == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
+        }
+        if (lane == 0) s_open[bq] = open;
+    }
+    __syncthreads();
+
+    // 4. the open blocks into the list (one atomic per tile), the open locations into shared memory
+    if (warp == 0) {
+        const int nb = a.sb * a.sb;
+        const int o = lane < nb ? s_open[lane] : 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, o);
+        int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(a.count_cur, __popc(bal));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (o) {
+            const int by = ty * a.sb + lane / a.sb, bx = tx * a.sb + lane % a.sb;
+            a.list[base + __popc(bal & ((1u << lane) - 1u))] = (int32_t)(((size_t)nn * a.nby + by) * a.nbx + bx);
+        }
+    }
+    for (int q = threadIdx.x; q < span * span; q += LT) {
+        const int li = q / span, lj = q - (q / span) * span;
+        if (s_open[(li / a.b) * a.sb + lj / a.b] && oy0 + li < a.Ho && ox0 + lj < a.Wo)
+            locs[atomicAdd(&s_nloc, 1)] = (li << 16) | lj;
+    }
+    __syncthreads();
+
+    // 5. w * r_t at the open locations into z (and y = act(z) when there is no shortcut)
+    const int M = s_nloc;
+    T* y = static_cast<T*>(a.y);
+    const bool y_here = y != nullptr && a.sc == nullptr;
+    if (DW) {
+        for (int it = threadIdx.x; it < M * a.C; it += LT) {
+            const int c = it % a.C, m = it / a.C;
+            const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
+            const float* r = R + (size_t)(li * a.stride * a.FW + lj * a.stride) * a.CP + c;
+            float acc = 0.f;
+            for (int kh = 0; kh < a.KH; ++kh)
+                for (int kw = 0; kw < a.KW; ++kw)
+                    acc = fmaf(__ldg(a.wcc + (size_t)(kh * a.KW + kw) * a.Co + c), r[(size_t)(kh * a.FW + kw) * a.CP],
+                               acc);
+            const size_t zo = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + c;
+            const float zv = a.z[zo] + acc;
+            a.z[zo] = zv;
+            if (y_here) y[zo] = from_f32<T>(activate(zv, a.act));
+        }
+    } else {
+        const int nq = (a.opg + 3) >> 2;             // output-channel quads per group
+        const int nm = (M + LPI - 1) / LPI;
+        const int items = nm * a.groups * nq;
+        for (int it = threadIdx.x; it < items; it += LT) {
+            const int q = it % nq;
+            const int rest = it / nq;
+            const int grp = rest % a.groups, mi = rest / a.groups;
+            const int o = grp * a.opg + q * 4;
+            const int oend = grp * a.opg + a.opg;
+            int rb[LPI];
+            long long zl[LPI];
+#pragma unroll
+            for (int u = 0; u < LPI; ++u) {
+                const int m = mi * LPI + u;
+                if (m < M) {
+                    const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
+                    rb[u] = (li * a.stride * a.FW + lj * a.stride) * a.CP + grp * a.cpg;
+                    zl[u] = ((long long)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj;
+                } else {
+                    rb[u] = 0;
+                    zl[u] = -1;
+                }
+            }
+            float acc[LPI][4];
+#pragma unroll
+            for (int u = 0; u < LPI; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
+            for (int kh = 0; kh < a.KH; ++kh) {
+                for (int kw = 0; kw < a.KW; ++kw) {
+                    const float* wr = a.wcc + (size_t)((kh * a.KW + kw) * a.cpg) * a.Co + o;
+                    const int toff = (kh * a.FW + kw) * a.CP;
+#pragma unroll 4
+                    for (int ci = 0; ci < a.cpg; ++ci) {
+                        float4 w;
+                        if (V4) {
+                            w = __ldg(reinterpret_cast<const float4*>(wr + (size_t)ci * a.Co));
+                        } else {
+                            const float* wp = wr + (size_t)ci * a.Co;
+                            w.x = __ldg(wp);
+                            w.y = o + 1 < oend ? __ldg(wp + 1) : 0.f;
+                            w.z = o + 2 < oend ? __ldg(wp + 2) : 0.f;
+                            w.w = o + 3 < oend ? __ldg(wp + 3) : 0.f;
+                        }
+#pragma unroll
+                        for (int u = 0; u < LPI; ++u) {
+                            const float r = R[rb[u] + toff + ci];
+                            acc[u][0] = fmaf(r, w.x, acc[u][0]);
+                            acc[u][1] = fmaf(r, w.y, acc[u][1]);
+                            acc[u][2] = fmaf(r, w.z, acc[u][2]);
+                            acc[u][3] = fmaf(r, w.w, acc[u][3]);
+                        }
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < LPI; ++u) {
+                if (zl[u] < 0) continue;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (o + j >= oend) continue;
+                    const size_t zo = (size_t)zl[u] * a.Co + o + j;
+                    const float zv = a.z[zo] + acc[u][j];
+                    a.z[zo] = zv;
+                    if (y_here) y[zo] = from_f32<T>(activate(zv, a.act));
+                }
+            }
+        }
+    }
+
+    // 6. with a shortcut: y = act(z + shortcut) over the tile's output locations
+    if (y != nullptr && a.sc != nullptr) {
+        __syncthreads();   // this CTA's z updates are visible to all its threads
+        const T* sc = static_cast<const T*>(a.sc);
+        const int th = min(span, a.Ho - oy0), tw = min(span, a.Wo - ox0);
+        for (int it = threadIdx.x; it < th * tw * a.Co; it += LT) {
+            const int c = it % a.Co, p = it / a.Co;
+            const size_t zo = (((size_t)nn * a.Ho + oy0 + p / tw) * a.Wo + ox0 + p % tw) * a.Co + c;
+            y[zo] = from_f32<T>(activate(a.z[zo] + to_f32(sc[zo]), a.act));
+        }
+    }
+}
+
+// ------------------------------------------------------------- staged form
+constexpr int FT = 256;                          // threads per CTA
+constexpr int SW = 32;                           // output channels per CTA (dense layers)
+constexpr int FLPI = 2;                          // output locations per work item
+constexpr uint64_t LOCAL_WAIT_NS = 1000000000ull;
+
+struct FastArgs {
+    const void* wpack;         // dense: [slice][K][SW]; depthwise: [taps][C] (layer dtype)
+    uint32_t wbytes;           // weight bytes of one CTA (a multiple of 16)
+    const void* xt;            // x_t and x_{t-1} in global memory (owned pixels outside the footprint)
+    const void* xp;
+    void* xn;
+    const uint8_t* chg_prev;
+    uint8_t* chg_cur;
+    float* z;
+    void* y;
+    const void* sc;
+    uint8_t* mask;
+    int32_t* list;
+    int32_t* count_cur;
+    int32_t* count_next;
+    int* err;
+    int force;
+    int n, H, W, C, Ho, Wo, Co, KH, KW, stride, pad, b, nby, nbx, act;
+    int sb, nty, ntx, FH, FW, CP, nsl, K;
+    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_red;   // byte offsets from the aligned base
+    float thr;
+};
+
+__device__ __forceinline__ float4 load_w4(const float* w) { return *reinterpret_cast<const float4*>(w); }
+__device__ __forceinline__ float4 load_w4(const __nv_bfloat16* w)
+{
+    const uint2 v = *reinterpret_cast<const uint2*>(w);
+    const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.x));
+    const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.y));
+    return make_float4(lo.x, lo.y, hi.x, hi.y);
+}
+
+// Residuals of one 16-byte chunk of a pixel (8 bf16 or 4 fp32 channels),
+// their l1 sum, and whether any bit differs.
+__device__ __forceinline__ int chunk_residual(const uint4& a, const uint4& b, float (&r)[8], __nv_bfloat16*)
+{
+    const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+    const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 fa = __bfloat1622float2(pa[k]), fb = __bfloat1622float2(pb[k]);
+        r[2 * k] = fa.x - fb.x;
+        r[2 * k + 1] = fa.y - fb.y;
+    }
+    return 8;
+}
+
+__device__ __forceinline__ int chunk_residual(const uint4& a, const uint4& b, float (&r)[8], float*)
+{
+    r[0] = __uint_as_float(a.x) - __uint_as_float(b.x);
+    r[1] = __uint_as_float(a.y) - __uint_as_float(b.y);
+    r[2] = __uint_as_float(a.z) - __uint_as_float(b.z);
+    r[3] = __uint_as_float(a.w) - __uint_as_float(b.w);
+    return 4;
+}
+
+__device__ __forceinline__ float2 load_pair(const float* p) { return *reinterpret_cast<const float2*>(p); }
+__device__ __forceinline__ float2 load_pair(const __nv_bfloat16* p)
+{
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+}
+__device__ __forceinline__ void store_pair(float* p, float a, float b) { *reinterpret_cast<float2*>(p) = make_float2(a, b); }
+__device__ __forceinline__ void store_pair(__nv_bfloat16* p, float a, float b)
+{
+    *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(a, b);
+}
+
+template <typename T, bool DW>
+__global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_constant__ CUtensorMap tm_xt,
+                                                               const __grid_constant__ CUtensorMap tm_xp,
+                                                               const FastArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t bars[2];    // 0: weights, 1: footprints
+    __shared__ int s_open[MAX_TILE_BLOCKS];
+    __shared__ int s_nloc;
+    uint8_t* base = align_smem_1024(smem_raw);
+    const T* Xt = reinterpret_cast<const T*>(base);
+    const T* Xp = reinterpret_cast<const T*>(base + a.off_xp);
+    const T* Ws = reinterpret_cast<const T*>(base + a.off_w);
+    float* R = reinterpret_cast<float*>(base + a.off_r);     // dense only: [FP][CP] residual
+    float* P = reinterpret_cast<float*>(base + a.off_p);
+    int* locs = reinterpret_cast<int*>(base + a.off_loc);
+    float* red = reinterpret_cast<float*>(base + a.off_red); // dense only: k-split partial sums
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    constexpr int NW = FT / 32;
+    const int sl = DW ? 0 : (int)(blockIdx.x % a.nsl);
+    const int tile = DW ? (int)blockIdx.x : (int)(blockIdx.x / a.nsl);
+    const int tx = tile % a.ntx, ty = (tile / a.ntx) % a.nty, nn = tile / (a.ntx * a.nty);
+    const int span = a.sb * a.b;
+    const int oy0 = ty * span, ox0 = tx * span;
+    const int fy0 = oy0 * a.stride - a.pad, fx0 = ox0 * a.stride - a.pad;
+    const int FP = a.FH * a.FW;
+    const uint32_t bar_w = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]);
+
+    if (tid == 0) {
+        mbar_init(bar_w, 1);
+        mbar_init(bar_x, 1);
+        fence_mbar_init();
+        // the weights are constant state: fetch them before waiting for the producer of x_t
+        mbar_arrive_expect_tx(bar_w, a.wbytes);
+        bulk_load(smem_u32(Ws), static_cast<const uint8_t*>(a.wpack) + (size_t)sl * a.wbytes, a.wbytes, bar_w);
+        prefetch_tmap(&tm_xt);
+        prefetch_tmap(&tm_xp);
+        s_nloc = 0;
+    }
+    grid_dependency_wait();
+    if (tid == 0) {
+        mbar_arrive_expect_tx(bar_x, 2u * (uint32_t)FP * (uint32_t)a.C * (uint32_t)sizeof(T));
+        tma_load_4d(smem_u32(Xt), &tm_xt, bar_x, 0, fx0, fy0, nn);
+        tma_load_4d(smem_u32(Xp), &tm_xp, bar_x, 0, fx0, fy0, nn);
+    }
+    grid_launch_dependents();
+    if (blockIdx.x == 0 && tid == 0) *a.count_next = 0;
+    __syncthreads();   // barrier initialisation visible before anyone waits on it
+    {
+        const bool ok = mbar_wait(bar_x, 0, nullptr, a.err, LOCAL_WAIT_NS);
+        if (!__syncthreads_and(ok)) {
+            // copies may still be in flight into this CTA's shared memory: wait for them (bounded) first
+            mbar_wait(bar_x, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            return;
+        }
+    }
+
+    // owned input pixels of this tile (every input pixel has exactly one owner tile)
+    const int own_y0 = min(ty * span * a.stride, a.H);
+    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
+    const int own_x0 = min(tx * span * a.stride, a.W);
+    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
+    T* xn = static_cast<T*>(a.xn);
+
+    // residuals, norms and (slice 0) the commit of owned pixels inside the footprint: G lanes per
+    // pixel, 16-byte chunks (a pixel is CH chunks)
+    {
+        constexpr int EPC = 16 / (int)sizeof(T);
+        const int CH = a.C / EPC;
+        int lg = 0;
+        while ((1 << lg) < CH && lg < 5) ++lg;
+        const int G = 1 << lg, gpw = 32 >> lg, sub = lane & (G - 1);
+        for (int q0 = warp * gpw; q0 < FP; q0 += NW * gpw) {
+            const int q = q0 + (lane >> lg);
+            const bool valid = q < FP;
+            const uint4* xs = reinterpret_cast<const uint4*>(Xt + (size_t)(valid ? q : 0) * a.C);
+            const uint4* ps = reinterpret_cast<const uint4*>(Xp + (size_t)(valid ? q : 0) * a.C);
+            float sum = 0.f;
+            unsigned d = 0;
+            if (valid) {
+                for (int k = sub; k < CH; k += G) {
+                    const uint4 av = xs[k], bv = ps[k];
+                    float r[8];
+                    const int ne = chunk_residual(av, bv, r, (T*)nullptr);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        if (e < ne) sum += fabsf(r[e]);
+                    d |= (av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w);
+                    if (!DW) {
+                        float4* rr = reinterpret_cast<float4*>(R + (size_t)q * a.CP + k * EPC);
+                        rr[0] = make_float4(r[0], r[1], r[2], r[3]);
+                        if (EPC == 8) rr[1] = make_float4(r[4], r[5], r[6], r[7]);
+                    }
+                }
+            }
+            for (int off = 1; off < G; off <<= 1) {
+                sum += __shfl_xor_sync(0xffffffffu, sum, off);
+                d |= __shfl_xor_sync(0xffffffffu, d, off);
+            }
+            if (valid && sub == 0) P[q] = sum;
+            if (sl == 0 && valid) {
+                const int iy = fy0 + q / a.FW, ix = fx0 + q % a.FW;
+                if (iy >= own_y0 && iy < own_y1 && ix >= own_x0 && ix < own_x1) {
+                    const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
+                    if (d || a.chg_prev[pix]) {
+                        uint4* dst = reinterpret_cast<uint4*>(xn) + pix * CH;
+                        for (int k = sub; k < CH; k += G) dst[k] = xs[k];
+                    }
+                    if (sub == 0) a.chg_cur[pix] = d ? 1 : 0;
+                }
+            }
+        }
+    }
+    // owned pixels outside the footprint (input rows or columns no output location reads)
+    if (sl == 0) {
+        const T* xt = static_cast<const T*>(a.xt);
+        const T* xp = static_cast<const T*>(a.xp);
+        const int ow = own_x1 - own_x0, npx = (own_y1 - own_y0) * ow;
+        for (int q = warp; q < npx; q += NW) {
+            const int iy = own_y0 + q / ow, ix = own_x0 + q % ow;
+            if (iy - fy0 < a.FH && ix - fx0 < a.FW) continue;   // done from the footprint
+            const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
+            unsigned d = 0;
+            for (int c = lane; c < a.C; c += 32) d |= bits_of(xt[pix * a.C + c]) ^ bits_of(xp[pix * a.C + c]);
+            const bool changed = __any_sync(0xffffffffu, d != 0);
+            if (changed || a.chg_prev[pix])
+                for (int c = lane; c < a.C; c += 32) xn[pix * a.C + c] = xt[pix * a.C + c];
+            if (lane == 0) a.chg_cur[pix] = changed ? 1 : 0;
+        }
+    }
+    __syncthreads();
+
+    // block gates of the tile (a warp per gate block)
+    for (int bq = warp; bq < a.sb * a.sb; bq += NW) {
+        const int bi = bq / a.sb, bj = bq - (bq / a.sb) * a.sb;
+        const int by = ty * a.sb + bi, bx = tx * a.sb + bj;
+        int open = 0;
+        if (by < a.nby && bx < a.nbx) {
+            const int bh = min(a.b, a.Ho - by * a.b), bw = min(a.b, a.Wo - bx * a.b);
+            float best = -1.f;
+            for (int q = lane; q < bh * bw; q += 32) {
+                const int li = bi * a.b + q / bw, lj = bj * a.b + q % bw;
+                float S = 0.f;
+                for (int kh = 0; kh < a.KH; ++kh)
+                    for (int kw = 0; kw < a.KW; ++kw) S += P[(li * a.stride + kh) * a.FW + lj * a.stride + kw];
+                best = fmaxf(best, S);
+            }
+            best = warp_max(best);
+            open = (a.force || best > a.thr) ? 1 : 0;
+            if (sl == 0 && lane == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
+        }
+        if (lane == 0) s_open[bq] = open;
+    }
+    __syncthreads();
+    if (sl == 0 && warp == 0) {
+        const int nb = a.sb * a.sb;
+        const int o = lane < nb ? s_open[lane] : 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, o);
+        int basei = 0;
+        if (lane == 0 && bal) basei = atomicAdd(a.count_cur, __popc(bal));
+        basei = __shfl_sync(0xffffffffu, basei, 0);
+        if (o) {
+            const int by = ty * a.sb + lane / a.sb, bx = tx * a.sb + lane % a.sb;
+            a.list[basei + __popc(bal & ((1u << lane) - 1u))] = (int32_t)(((size_t)nn * a.nby + by) * a.nbx + bx);
+        }
+    }
+    for (int q = tid; q < span * span; q += FT) {
+        const int li = q / span, lj = q - (q / span) * span;
+        if (s_open[(li / a.b) * a.sb + lj / a.b] && oy0 + li < a.Ho && ox0 + lj < a.Wo)
+            locs[atomicAdd(&s_nloc, 1)] = (li << 16) | lj;
+    }
+    {
+        const bool ok = mbar_wait(bar_w, 0, nullptr, a.err, LOCAL_WAIT_NS);
+        if (!__syncthreads_and(ok)) {
+            mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            return;
+        }
+    }
+
+    const int M = s_nloc;
+    T* y = static_cast<T*>(a.y);
+    const bool y_here = y != nullptr && a.sc == nullptr;
+    if (DW) {
+        // a thread per channel pair (weights in registers) and a share of the open locations
+        const int NCP = a.C / 2, ngrp = FT / NCP;
+        const int cp = tid % NCP, g = tid / NCP, c = 2 * cp;
+        float2 wreg[9];   // 3x3 layers: the channel pair's weights
+#pragma unroll
+        for (int tp = 0; tp < 9; ++tp)
+            wreg[tp] = (a.KH == 3 && a.KW == 3) ? load_pair(Ws + tp * a.C + c) : make_float2(0.f, 0.f);
+        if (g < ngrp) {
+            for (int m = g; m < M; m += ngrp) {
+                const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
+                const int p0 = li * a.stride * a.FW + lj * a.stride;
+                const size_t zo = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + c;
+                const float2 zold = *reinterpret_cast<const float2*>(a.z + zo);
+                float acc0 = 0.f, acc1 = 0.f;
+                if (a.KH == 3 && a.KW == 3) {
+#pragma unroll
+                    for (int kh = 0; kh < 3; ++kh)
+#pragma unroll
+                        for (int kw = 0; kw < 3; ++kw) {
+                            const size_t e = (size_t)(p0 + kh * a.FW + kw) * a.C + c;
+                            const float2 xa = load_pair(Xt + e), xb = load_pair(Xp + e);
+                            acc0 = fmaf(wreg[kh * 3 + kw].x, xa.x - xb.x, acc0);
+                            acc1 = fmaf(wreg[kh * 3 + kw].y, xa.y - xb.y, acc1);
+                        }
+                } else {
+                    for (int kh = 0; kh < a.KH; ++kh)
+                        for (int kw = 0; kw < a.KW; ++kw) {
+                            const size_t e = (size_t)(p0 + kh * a.FW + kw) * a.C + c;
+                            const float2 xa = load_pair(Xt + e), xb = load_pair(Xp + e);
+                            const float2 w = load_pair(Ws + (kh * a.KW + kw) * a.C + c);
+                            acc0 = fmaf(w.x, xa.x - xb.x, acc0);
+                            acc1 = fmaf(w.y, xa.y - xb.y, acc1);
+                        }
+                }
+                const float z0 = zold.x + acc0, z1 = zold.y + acc1;
+                *reinterpret_cast<float2*>(a.z + zo) = make_float2(z0, z1);
+                if (y_here) store_pair(y + zo, activate(z0, a.act), activate(z1, a.act));
+            }
+        }
+    } else {
+        constexpr int NQ = SW / 4;
+        const int items = (M + FLPI - 1) / FLPI * NQ;
+        const int parts = items == 0 ? 1 : max(1, min(8, FT / items));
+        const int o_base = sl * SW;
+        // pre: also load the item's z values now, so that their latency hides behind the contraction
+        auto contract = [&](int item, int k_lo, int k_hi, float (&acc)[FLPI][4], long long (&zl)[FLPI],
+                            float (&zv)[FLPI][4], bool pre) {
+            const int q = item % NQ, mi = item / NQ;
+            const int o = o_base + q * 4;
+            int rb[FLPI];
+#pragma unroll
+            for (int u = 0; u < FLPI; ++u) {
+                const int m = mi * FLPI + u;
+                if (m < M) {
+                    const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
+                    rb[u] = (li * a.stride * a.FW + lj * a.stride) * a.CP;
+                    zl[u] = ((long long)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj;
+                } else {
+                    rb[u] = 0;
+                    zl[u] = -1;
+                }
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    acc[u][j] = 0.f;
+                    zv[u][j] = (pre && zl[u] >= 0 && o + j < a.Co) ? a.z[(size_t)zl[u] * a.Co + o + j] : 0.f;
+                }
+            }
+            // k = tap * C + ci; walk the taps of [k_lo, k_hi)
+            int tap = k_lo / a.C, ci = k_lo - tap * a.C;
+            int k = k_lo;
+            while (k < k_hi) {
+                const int kh = tap / a.KW, kw = tap - (tap / a.KW) * a.KW;
+                const int toff = (kh * a.FW + kw) * a.CP;
+                const int cend = min(a.C, ci + (k_hi - k));
+                const T* wr = Ws + (size_t)(tap * a.C) * SW + q * 4;
+#pragma unroll 4
+                for (int c = ci; c < cend; ++c) {
+                    const float4 w = load_w4(wr + (size_t)c * SW);
+#pragma unroll
+                    for (int u = 0; u < FLPI; ++u) {
+                        const float r = R[rb[u] + toff + c];
+                        acc[u][0] = fmaf(r, w.x, acc[u][0]);
+                        acc[u][1] = fmaf(r, w.y, acc[u][1]);
+                        acc[u][2] = fmaf(r, w.z, acc[u][2]);
+                        acc[u][3] = fmaf(r, w.w, acc[u][3]);
+                    }
+                }
+                k += cend - ci;
+                ci = 0;
+                ++tap;
+            }
+        };
+        auto store = [&](int item, const float (&acc)[FLPI][4], const long long (&zl)[FLPI],
+                         const float (&zv)[FLPI][4]) {
+            const int o = o_base + (item % NQ) * 4;
+#pragma unroll
+            for (int u = 0; u < FLPI; ++u) {
+                if (zl[u] < 0) continue;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if (o + j >= a.Co) continue;
+                    const size_t zo = (size_t)zl[u] * a.Co + o + j;
+                    const float znew = zv[u][j] + acc[u][j];
+                    a.z[zo] = znew;
+                    if (y_here) y[zo] = from_f32<T>(activate(znew, a.act));
+                }
+            }
+        };
+        if (parts == 1) {
+            for (int it = tid; it < items; it += FT) {
+                float acc[FLPI][4], zv[FLPI][4];
+                long long zl[FLPI];
+                contract(it, 0, a.K, acc, zl, zv, true);
+                store(it, acc, zl, zv);
+            }
+        } else {
+            // too few open locations to occupy the CTA: split k over `parts` thread groups
+            const int item = tid % items, part = tid / items;
+            float acc[FLPI][4], zv[FLPI][4];
+            long long zl[FLPI];
+            if (part < parts) {
+                const int k_lo = (int)((long long)a.K * part / parts), k_hi = (int)((long long)a.K * (part + 1) / parts);
+                contract(item, k_lo, k_hi, acc, zl, zv, part == 0);
+                if (part > 0) {
+#pragma unroll
+                    for (int u = 0; u < FLPI; ++u)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) red[((part - 1) * items + item) * (FLPI * 4) + u * 4 + j] = acc[u][j];
+                }
+            }
+            __syncthreads();
+            if (part == 0) {
+                for (int pp = 1; pp < parts; ++pp)
+#pragma unroll
+                    for (int u = 0; u < FLPI; ++u)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) acc[u][j] += red[((pp - 1) * items + item) * (FLPI * 4) + u * 4 + j];
+                store(item, acc, zl, zv);
+            }
+        }
+    }
+
+    if (y != nullptr && a.sc != nullptr) {
+        __syncthreads();
+        const T* sc = static_cast<const T*>(a.sc);
+        const int th = min(span, a.Ho - oy0), tw = min(span, a.Wo - ox0);
+        const int c0 = DW ? 0 : sl * SW, nc = DW ? a.Co : min(SW, a.Co - sl * SW);
+        for (int it = tid; it < th * tw * nc; it += FT) {
+            const int c = c0 + it % nc, p = it / nc;
+            const size_t zo = (((size_t)nn * a.Ho + oy0 + p / tw) * a.Wo + ox0 + p % tw) * a.Co + c;
+            y[zo] = from_f32<T>(activate(a.z[zo] + to_f32(sc[zo]), a.act));
+        }
+    }
+}
+
+// Weights of the staged form, in the layer's dtype: dense [slice][K][SW]
+// (K index = tap * c_in + ci, channels past c_out zero), depthwise [taps][C].
+template <typename T>
+__global__ void pack_local_weights_kernel(const float* __restrict__ wcc, T* __restrict__ out, int K, int Co,
+                                          int nsl, int dw)
+{
+    const long long total = dw ? (long long)K * Co : (long long)nsl * K * SW;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        if (dw) {
+            out[i] = from_f32<T>(wcc[i]);
+        } else {
+            const int j = (int)(i % SW);
+            const long long rest = i / SW;
+            const int k = (int)(rest % K), sl = (int)(rest / K);
+            const int o = sl * SW + j;
+            out[i] = from_f32<T>(o < Co ? wcc[(size_t)k * Co + o] : 0.f);
+        }
+    }
+}
+
+struct LocalShape {
+    int sb, span, FH, FW, CP;
+    size_t smem;
+};
+
+LocalShape local_shape(const Layer& L, int sb)
+{
+    LocalShape s;
+    s.sb = sb;
+    s.span = sb * L.p.block;
+    s.FH = (s.span - 1) * L.p.stride + L.p.k_h;
+    s.FW = (s.span - 1) * L.p.stride + L.p.k_w;
+    s.CP = L.p.c_in | 1;   // odd pixel stride: neighbouring locations fall in different banks
+    const size_t fp = (size_t)s.FH * s.FW;
+    s.smem = (fp * s.CP + fp + (size_t)s.span * s.span) * sizeof(float);
+    return s;
+}
+
+LocalShape choose_shape(const Layer& L)
+{
+    int sb = L.p.block >= 4 ? 1 : (4 + L.p.block - 1) / L.p.block;
+    LocalShape s = local_shape(L, sb);
+    while (s.smem > LOCAL_MAX_SMEM && sb > 1) s = local_shape(L, --sb);
+    return s;
+}
+
+template <typename T>
+const void* kernel_of(const Layer& L)
+{
+    if (L.cpg == 1 && L.opg == 1) return (const void*)step_local_kernel<T, true, false>;
+    if (L.p.c_out % 4 == 0 && L.opg % 4 == 0) return (const void*)step_local_kernel<T, false, true>;
+    return (const void*)step_local_kernel<T, false, false>;
+}
+
+const void* kernel_of(const Layer& L)
+{
+    return L.p.dtype == SKIPCONV_BF16 ? kernel_of<__nv_bfloat16>(L) : kernel_of<float>(L);
+}
+
+// ------------------------------------------------------ staged form, host side
+struct StagedShape {
+    LocalShape g;
+    int nsl;
+    uint32_t wbytes;
+    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_red;
+    size_t smem;
+};
+
+inline uint32_t up128(size_t v) { return (uint32_t)((v + 127) & ~(size_t)127); }
+
+bool is_depthwise(const Layer& L) { return L.cpg == 1 && L.opg == 1; }
+
+StagedShape staged_shape(const Layer& L, int sb)
+{
+    StagedShape t;
+    t.g = local_shape(L, sb);
+    t.g.CP = L.p.c_in + 4;   // 16-byte aligned residual rows, consecutive pixels 4 banks apart
+    const bool dw = is_depthwise(L);
+    const size_t fp = (size_t)t.g.FH * t.g.FW;
+    const int K = L.p.k_h * L.p.k_w * L.p.c_in;
+    t.nsl = dw ? 1 : (L.p.c_out + SW - 1) / SW;
+    const size_t wb = dw ? (size_t)L.p.k_h * L.p.k_w * L.p.c_in * L.esize : (size_t)K * SW * L.esize;
+    t.wbytes = (uint32_t)((wb + 15) & ~(size_t)15);
+    const uint32_t xb = up128(fp * L.p.c_in * L.esize);
+    t.off_xp = xb;
+    t.off_w = 2 * xb;
+    t.off_r = t.off_w + up128(t.wbytes);
+    t.off_p = t.off_r + (dw ? 0 : up128(fp * t.g.CP * sizeof(float)));
+    t.off_loc = t.off_p + up128(fp * sizeof(float));
+    t.off_red = t.off_loc + up128((size_t)t.g.span * t.g.span * sizeof(int));
+    t.smem = (size_t)t.off_red + (dw ? 0 : up128((size_t)FT * FLPI * 4 * sizeof(float))) + 1024;
+    return t;
+}
+
+// The staged form needs TMA boxes of the footprint (a pixel's channels a
+// multiple of 16 bytes, every box edge at most 256) and a dense (groups = 1)
+// or depthwise layer.
+bool staged_ok(const Layer& L, StagedShape* out)
+{
+    if (!(L.p.groups == 1 || is_depthwise(L))) return false;
+    if ((L.p.c_in * L.esize) % 16 || L.p.c_in > 256) return false;
+    int sb = L.p.block >= 4 ? 1 : (4 + L.p.block - 1) / L.p.block;
+    StagedShape t = staged_shape(L, sb);
+    while (t.smem > LOCAL_MAX_SMEM && sb > 1) t = staged_shape(L, --sb);
+    if (t.smem > LOCAL_MAX_SMEM || t.g.FH > 256 || t.g.FW > 256) return false;
+    if ((long long)L.p.n_streams * ((L.nby + sb - 1) / sb) * ((L.nbx + sb - 1) / sb) * t.nsl > 0x7fffffffLL)
+        return false;
+    if (out) *out = t;
+    return true;
+}
+
+bool encode_footprint_map(CUtensorMap* m, const void* base, const Layer& L, const StagedShape& t)
+{
+    EncodeTiledFn enc = encode_tiled_fn();
+    if (!enc) return false;
+    const cuuint64_t C = L.p.c_in, W = L.p.w, H = L.p.h, N = L.p.n_streams, es = L.esize;
+    cuuint64_t dims[4] = {C, W, H, N};
+    cuuint64_t strides[3] = {C * es, W * C * es, H * W * C * es};
+    cuuint32_t box[4] = {(cuuint32_t)C, (cuuint32_t)t.g.FW, (cuuint32_t)t.g.FH, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUtensorMapDataType dt =
+        L.p.dtype == SKIPCONV_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    return enc(m, dt, 4, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+const void* staged_kernel_of(const Layer& L)
+{
+    const bool dw = is_depthwise(L);
+    if (L.p.dtype == SKIPCONV_BF16)
+        return dw ? (const void*)step_local_staged_kernel<__nv_bfloat16, true>
+                  : (const void*)step_local_staged_kernel<__nv_bfloat16, false>;
+    return dw ? (const void*)step_local_staged_kernel<float, true> : (const void*)step_local_staged_kernel<float, false>;
+}
+
+cudaLaunchConfig_t pdl_config(const Layer& L, long long grid, int threads, size_t smem, cudaLaunchAttribute* attr)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = L.stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cfg;
+}
+
+}  // namespace
+
+bool step_local_preferred(const Layer& L)
+{
+    if (L.p.gate == SKIPCONV_GATE_GUMBEL || L.p.dense_mode) return false;
+    const double dense_macs = (double)L.p.n_streams * L.ho * L.wo * L.p.c_out * L.cpg * L.p.k_h * L.p.k_w;
+    return dense_macs <= LOCAL_AUTO_MAX_MACS && staged_ok(L, nullptr);
+}
+
+bool step_local_supported(const Layer& L)
+{
+    if (L.path != SKIPCONV_PATH_CUDA_CORE || L.p.conv_path == SKIPCONV_PATH_CUDA_CORE_SEPARATE) return false;
+    if (L.p.gate == SKIPCONV_GATE_GUMBEL) return false;
+    return staged_ok(L, nullptr) || choose_shape(L).smem <= LOCAL_MAX_SMEM;
+}
+
+cudaError_t step_local_prepare(Layer& L)
+{
+    StagedShape t;
+    if (staged_ok(L, &t)) {
+        if (!encode_footprint_map(&L.tmap_fp[0], L.xbuf[0], L, t) || !encode_footprint_map(&L.tmap_fp[1], L.xbuf[1], L, t)) {
+            set_error("tensor map of the state frames rejected");
+            return cudaErrorInvalidValue;
+        }
+        const size_t bytes = (size_t)t.wbytes * t.nsl;
+        cudaError_t e = cudaMalloc(&L.w_loc, bytes);
+        if (e != cudaSuccess) {
+            L.w_loc = nullptr;
+            return e;
+        }
+        L.state_bytes += bytes;
+        e = cudaMemsetAsync(L.w_loc, 0, bytes, L.stream);
+        if (e != cudaSuccess) return e;
+        const bool dw = is_depthwise(L);
+        const int K = L.p.k_h * L.p.k_w * L.p.c_in;
+        const long long total = dw ? (long long)K * L.p.c_out : (long long)t.nsl * K * SW;
+        const int grid = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
+        if (L.p.dtype == SKIPCONV_BF16)
+            pack_local_weights_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(
+                L.w_cc, (__nv_bfloat16*)L.w_loc, dw ? L.p.k_h * L.p.k_w : K, L.p.c_out, t.nsl, dw ? 1 : 0);
+        else
+            pack_local_weights_kernel<float><<<grid, 256, 0, L.stream>>>(L.w_cc, (float*)L.w_loc,
+                                                                         dw ? L.p.k_h * L.p.k_w : K, L.p.c_out,
+                                                                         t.nsl, dw ? 1 : 0);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        L.local_staged = 1;
+        return ensure_dynamic_smem(staged_kernel_of(L), t.smem);
+    }
+    L.local_staged = 0;
+    return ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
+}
+
+cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* shortcut, int force)
+{
+    const int cur = (int)(L.t & 1), nxt = cur ^ 1;
+    cudaLaunchAttribute attr[1];
+    if (L.local_staged) {
+        StagedShape t;
+        if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
+        alignas(64) CUtensorMap tm_xt;
+        if (!encode_footprint_map(&tm_xt, x_t, L, t)) {
+            set_error("tensor map of x_t rejected");
+            return cudaErrorInvalidValue;
+        }
+        FastArgs a;
+        a.wpack = L.w_loc;
+        a.wbytes = t.wbytes;
+        a.xt = x_t;
+        a.xp = L.xbuf[cur];
+        a.xn = L.xbuf[nxt];
+        a.chg_prev = L.chg[nxt];
+        a.chg_cur = L.chg[cur];
+        a.z = L.z;
+        a.y = L.y;
+        a.sc = L.y ? shortcut : nullptr;
+        a.mask = L.mask;
+        a.list = L.list;
+        a.count_cur = step_count(L);
+        a.count_next = next_count(L);
+        a.err = L.err_dev;
+        a.force = force;
+        a.n = L.p.n_streams; a.H = L.p.h; a.W = L.p.w; a.C = L.p.c_in; a.Ho = L.ho; a.Wo = L.wo;
+        a.Co = L.p.c_out; a.KH = L.p.k_h; a.KW = L.p.k_w; a.stride = L.p.stride; a.pad = L.p.pad; a.b = L.p.block;
+        a.nby = L.nby; a.nbx = L.nbx; a.act = L.p.activation;
+        a.sb = t.g.sb;
+        a.nty = (L.nby + t.g.sb - 1) / t.g.sb;
+        a.ntx = (L.nbx + t.g.sb - 1) / t.g.sb;
+        a.FH = t.g.FH; a.FW = t.g.FW; a.CP = t.g.CP; a.nsl = t.nsl; a.K = L.p.k_h * L.p.k_w * L.p.c_in;
+        a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
+        a.off_red = t.off_red;
+        a.thr = L.gate_thr;
+        const long long grid = (long long)a.n * a.nty * a.ntx * t.nsl;
+        cudaLaunchConfig_t cfg = pdl_config(L, grid, FT, t.smem, attr);
+        const CUtensorMap* tm_xp = &L.tmap_fp[cur];
+        void* args[] = {&tm_xt, const_cast<CUtensorMap*>(tm_xp), &a};
+        return cudaLaunchKernelExC(&cfg, staged_kernel_of(L), args);
+    }
+    const LocalShape s = choose_shape(L);
+    LocalArgs a;
+    a.xt = x_t;
+    a.xp = L.xbuf[cur];
+    a.xn = L.xbuf[nxt];
+    a.chg_prev = L.chg[nxt];
+    a.chg_cur = L.chg[cur];
+    a.wcc = L.w_cc;
+    a.z = L.z;
+    a.y = L.y;
+    a.sc = L.y ? shortcut : nullptr;
+    a.mask = L.mask;
+    a.list = L.list;
+    a.count_cur = step_count(L);
+    a.count_next = next_count(L);
+    a.force = force;
+    a.n = L.p.n_streams; a.H = L.p.h; a.W = L.p.w; a.C = L.p.c_in; a.Ho = L.ho; a.Wo = L.wo; a.Co = L.p.c_out;
+    a.KH = L.p.k_h; a.KW = L.p.k_w; a.stride = L.p.stride; a.pad = L.p.pad; a.b = L.p.block;
+    a.nby = L.nby; a.nbx = L.nbx; a.cpg = L.cpg; a.opg = L.opg; a.groups = L.p.groups; a.act = L.p.activation;
+    a.sb = s.sb;
+    a.nty = (L.nby + s.sb - 1) / s.sb;
+    a.ntx = (L.nbx + s.sb - 1) / s.sb;
+    a.FH = s.FH; a.FW = s.FW; a.CP = s.CP;
+    a.thr = L.gate_thr;
+    const long long tiles = (long long)a.n * a.nty * a.ntx;
+    if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = pdl_config(L, tiles, LT, s.smem, attr);
+    void* args[] = {&a};
+    return cudaLaunchKernelExC(&cfg, kernel_of(L), args);
+}
+
+}  // namespace sc

@@ -11,7 +11,8 @@ import ctypes
 
 from . import _lib
 from ._lib import (ACT_NONE, ACT_RELU, ACT_SILU, BF16, F32, GATE_GUMBEL, GATE_INPUT_MEAN, GATE_INPUT_SUM,  # noqa: F401
-                   GATE_OUTPUT, PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE, PATH_TENSOR_CORE_SEPARATE, Info,
+                   GATE_OUTPUT, PATH_AUTO, PATH_CUDA_CORE, PATH_CUDA_CORE_SEPARATE, PATH_TENSOR_CORE,
+                   PATH_TENSOR_CORE_SEPARATE, Info,
                    Params, SkipConvError, check)
 
 
@@ -106,7 +107,7 @@ def skipconv_profile(handle: int, enable: bool) -> None:
 
 def skipconv_profile_read(handle: int):
     """Returns (launches, ms), lists of PROFILE_KINDS per kernel kind: gate_pixel, gate_block, conv,
-    y_refresh, fused step."""
+    y_refresh, fused tensor-core step, one-launch CUDA-core step."""
     launches = (ctypes.c_longlong * _lib.PROFILE_KINDS)()
     ms = (ctypes.c_double * _lib.PROFILE_KINDS)()
     check("skipconv_profile_read", _lib.lib().skipconv_profile_read(handle, launches, ms))

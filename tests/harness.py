@@ -99,7 +99,8 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
                      phi_bias=0.0):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record and the conv path used.
-    expect_fused: None, or whether the layer must run as one fused launch.
+    expect_fused: None, or the info.fused value the layer must report (0 separate
+    launches, 1 one cooperative tensor-core launch, 2 one CUDA-core launch).
     reset_at: frames before which both sides are reset; ref_reset_at: frames
     before which only the oracle is reset (the GPU layer resets itself through
     key_interval)."""

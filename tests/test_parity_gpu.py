@@ -10,10 +10,12 @@ from oracle import GATE_INPUT_SUM, GATE_OUTPUT, LayerSpec
 
 pytestmark = pytest.mark.gpu
 
-AUTO, CUDA_CORE, TENSOR_CORE, SEPARATE = 0, 1, 2, 3
-# AUTO runs these bf16 8x8-block layers as one fused launch per step; SEPARATE
-# forces the gate and the tensor-core convolution into their own launches.
-FUSED = {AUTO: True, SEPARATE: False, CUDA_CORE: False}
+AUTO, CUDA_CORE, TENSOR_CORE, SEPARATE, CC_SEPARATE = 0, 1, 2, 3, 4
+# AUTO runs these bf16 8x8-block layers as one cooperative tensor-core launch
+# per step (fused = 1); SEPARATE forces the gate and the tensor-core
+# convolution into their own launches; CUDA_CORE runs the step as one
+# CUDA-core launch (fused = 2) and CC_SEPARATE as gate passes + convolution.
+FUSED = {AUTO: 1, SEPARATE: 0, CUDA_CORE: 2, CC_SEPARATE: 0}
 
 
 def spec_of(wl, li=0, **kw):
@@ -32,14 +34,16 @@ def frames_of(wl):
 
 
 # ----------------------------------------------------------- the workloads
-def test_c0_fp32_pixel_gates():
+@pytest.mark.parametrize("path", [AUTO, CC_SEPARATE])
+def test_c0_fp32_pixel_gates(path):
     wl = synth.make_workload("c0")
-    cmp, path = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "f32", name="c0")
-    assert path == CUDA_CORE and cmp.frames == 8
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "f32", name="c0",
+                                 conv_path=path, expect_fused=2 if path == AUTO else 0)
+    assert used == CUDA_CORE and cmp.frames == 8
     assert cmp.max_err <= 1e-4
 
 
-@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_c1_bf16_8x8_blocks(path):
     wl = synth.make_workload("c1")
     cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
@@ -56,20 +60,57 @@ def test_c1_streaming_tensor_core_kernel_with_y():
     assert used == TENSOR_CORE and cmp.frames == 16
 
 
-def test_c2_pose_stack_teacher_forced():
+@pytest.mark.parametrize("path", [AUTO, CC_SEPARATE])
+def test_c2_pose_stack_teacher_forced(path):
     wl = synth.make_workload("c2")
-    cmps, paths = run_stack_teacher_forced(wl)
+    cmps, paths = run_stack_teacher_forced(wl, conv_path=path)
     assert all(c.frames == 32 for c in cmps)
 
 
-def test_c3_mbconv_stack_teacher_forced():
+@pytest.mark.parametrize("path", [AUTO, CC_SEPARATE])
+def test_c3_mbconv_stack_teacher_forced(path):
     wl = synth.make_workload("c3")
-    cmps, paths = run_stack_teacher_forced(wl)
+    cmps, paths = run_stack_teacher_forced(wl, conv_path=path)
     assert all(c.frames == 32 for c in cmps)
+
+
+LOCAL_CASES = [
+    # name, n, h, w, c_in, c_out, k, stride, pad, groups, block, dtype
+    ("f32_b1_ragged", 2, 19, 23, 8, 12, 3, 1, 1, 1, 1, "f32"),
+    ("bf16_b3_stride2_ragged", 1, 37, 29, 16, 24, 3, 2, 1, 1, 3, "bf16"),
+    ("bf16_groups2", 1, 24, 20, 16, 32, 3, 1, 1, 2, 4, "bf16"),
+    ("bf16_depthwise_ragged", 1, 30, 26, 24, 24, 3, 1, 1, 24, 8, "bf16"),
+    ("bf16_cout6", 1, 20, 20, 8, 6, 3, 1, 1, 1, 4, "bf16"),
+    ("f32_k5_pad2_b2", 1, 21, 17, 4, 8, 5, 1, 2, 1, 2, "f32"),
+    ("bf16_1x1_b16", 1, 40, 36, 12, 20, 1, 1, 0, 1, 16, "bf16"),
+]
+
+
+@pytest.mark.parametrize("case", LOCAL_CASES, ids=[c[0] for c in LOCAL_CASES])
+@pytest.mark.parametrize("path", [CUDA_CORE, CC_SEPARATE])
+def test_cuda_core_geometries(case, path):
+    """CUDA-core layers in both forms (one launch per step, a CTA per tile of
+    gate blocks; or the separate gate and convolution launches): block sizes
+    1-16 (tiles of several blocks, ragged edge tiles), stride 2, 5x5 with
+    padding 2, 1x1, grouped and depthwise layers, c_out not a multiple of 4;
+    z, y, masks and the committed x_{t-1} every frame."""
+    name, n, h, w, c_in, c_out, k, stride, pad, groups, block, dtype = case
+    rng = np.random.default_rng(900 + block)
+    v = np.stack([synth.moving_squares_video(61 + s, 6, h, w, c_in, n_squares=2, size=6, speed=2, noise_std=0.01)
+                  for s in range(n)], axis=1)
+    frames = synth.round_to_bf16(v) if dtype == "bf16" else v.astype(np.float32)
+    wts = synth.he_weights(rng, c_out, c_in // groups, k, bf16=dtype == "bf16")
+    b = (rng.standard_normal(c_out) * 0.1).astype(np.float32)
+    b = synth.round_to_bf16(b) if dtype == "bf16" else b
+    spec = LayerSpec(n=n, c_in=c_in, c_out=c_out, h=h, w=w, k=k, stride=stride, pad=pad, groups=groups,
+                     block=block, eps=0.05)
+    cmp, used = run_single_layer(spec, wts, b, [frames[t] for t in range(6)], dtype, conv_path=path,
+                                 name=name, emit_y=True, expect_fused=FUSED[path])
+    assert used == CUDA_CORE and cmp.frames == 6
 
 
 @pytest.mark.parametrize("density", [0.0, 0.1, 0.5, 1.0])
-@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_c4_density_small(density, path):
     """c4's generator at a small size (2 streams, 32x40, 64 channels), 32 frames."""
     wl = synth.make_workload("c4", density=density, T=32, n=2, h=32, w=40, c=64)
@@ -78,7 +119,7 @@ def test_c4_density_small(density, path):
     assert cmp.frames == 32
 
 
-@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_ragged_tail_and_several_tiles(path):
     """Frame sizes that are not multiples of the block (ragged edge blocks)."""
     frames = synth.round_to_bf16(synth.moving_squares_video(77, 6, 100, 76, 64, n_squares=4, size=12))
@@ -91,7 +132,7 @@ def test_ragged_tail_and_several_tiles(path):
     assert cmp.frames == 6
 
 
-@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_dense_mode_is_dense_conv(path):
     wl = synth.make_workload("c1", T=4)
     cmp, _ = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
@@ -118,7 +159,7 @@ def test_reset_mid_sequence_and_single_frame():
     assert cmp.frames == 1
 
 
-@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_key_interval_resets_like_the_oracle(path):
     """key_interval = 3: steps 3 and 6 are key frames (Table 4's periodic
     reset), i.e. the oracle reset before frames 3 and 6."""
@@ -155,7 +196,7 @@ def test_gumbel_gate(case, path):
     spec = LayerSpec(n=n, c_in=c_in, c_out=c_out, h=h, w=w, k=3, stride=stride, pad=1, block=block, eps=0.0,
                      gate=GATE_GUMBEL)
     cmp, _ = run_single_layer(spec, wts, None, [frames[t] for t in range(5)], dtype, conv_path=path,
-                              name="gumbel " + name, phi=phi, phi_bias=-0.3, expect_fused=False)
+                              name="gumbel " + name, phi=phi, phi_bias=-0.3, expect_fused=0)
     assert cmp.frames == 5
 
 
