@@ -58,6 +58,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the single-layer and stacked workloads (c0-c3)")
+    ap.add_argument("--workloads-only", default=None, metavar="NAMES",
+                    help="run only these of the single-layer and stacked workloads (comma-separated, e.g. c2,c3) "
+                         "and print their report; for profiling them")
     ap.add_argument("--no-flush", action="store_true",
                     help="no L2 flush between timed steps: each step streams 134 MB of frames, more than the L2")
     ap.add_argument("--no-soak", action="store_true",
@@ -218,6 +221,8 @@ def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
 
 
 CONV_PATH = {"fused": 0, "separate": 3}   # AUTO (one fused launch per step) / TENSOR_CORE_SEPARATE
+LAUNCH_FORMS = {0: "separate gate and convolution launches", 1: "one cooperative tensor-core launch",
+                2: "one CUDA-core launch (a CTA per tile of gate blocks)"}
 
 
 GATES = {"input": 0, "output": 2}         # Input-Norm (mean), Output-Norm
@@ -435,7 +440,7 @@ def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c
             per_layer.append({"layer": L.name, "shape": "%dx%dx%d -> %dx%dx%d, k%d s%d g%d, b%d" % (
                 h_, w_, L.c_in, ho, wo, L.c_out, L.k, L.stride, L.groups, L.block),
                 "path": {1: "cuda-core", 2: "tensor-core"}.get(lays[li].info.conv_path),
-                "fused": bool(lays[li].info.fused), "launches": layer_launches[li],
+                "step_launch": LAUNCH_FORMS.get(lays[li].info.fused), "launches": layer_launches[li],
                 "open_location_density": loc / (wl.n * ho * wo), "kernel_us": layer_ms[li] * 1e3,
                 "eff_tflops": fl / (layer_ms[li] * 1e-3) / 1e12 if layer_ms[li] else None,
                 "roofline_frac": tr / (layer_ms[li] * 1e-3) if layer_ms[li] else None})
@@ -549,6 +554,14 @@ def main():
     pk, pk_src = peaks()
     hbm, tc_peak = pk["hbm_gbs"], pk["bf16_tflops"]
 
+    if args.workloads_only:
+        flush = None if args.no_flush else torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+        rep = workloads_report(torch, flush, tc_peak, hbm, names=tuple(args.workloads_only.split(",")))
+        if rank == 0:
+            print(json.dumps({"other_workloads": rep}), flush=True)
+        ranks.close()
+        return 0
+
     n_frames = args.warmup + args.steps + 1
     wl, frames, changed = device_frames(args.density, n_frames, rank, torch)
     flush = None if args.no_flush else torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
@@ -615,7 +628,7 @@ def main():
             "config": workload_config(args.density, flushed=not args.no_flush, gate=args.gate,
                                       key_interval=args.key_interval),
             "conv_path": {1: "cuda-core", 2: "tensor-core"}.get(info.conv_path),
-            "step_launches": "one fused launch" if info.fused else "separate gate and convolution launches",
+            "step_launches": LAUNCH_FORMS.get(info.fused),
             "active_blocks_per_step": active, "block_density_measured": active / (N_STREAMS * (H // BLOCK) ** 2),
             "changed_pixels_per_step": chg,
             "eff_tflops": flops / t_step / 1e12,

@@ -81,6 +81,7 @@ struct Layer {
     // one-launch CUDA-core step (sc_step_local.cu)
     int local_staged;       // 1: its TMA-footprint / staged-weight form
     CUtensorMap tmap_fp[2]; // footprint boxes of the two state frames
+    CUtensorMap tmap_ztile; // tile boxes of z
     void* w_loc;            // weights packed per CTA slice, layer dtype
 };
 
@@ -126,7 +127,7 @@ cudaError_t launch_step_fused(Layer& L, const void* x_t, int force);
 // One-launch step for CUDA-core layers (sc_step_local.cu): a CTA per tile of
 // gate blocks computes residual, norms, gates, convolution, y and the commit
 // from its own input footprint.
-constexpr size_t LOCAL_MAX_SMEM = 200 * 1024;
+constexpr size_t LOCAL_MAX_SMEM = 226 * 1024;
 // Layers whose dense step is at most this many MACs run on this form under
 // SKIPCONV_PATH_AUTO even where tensor cores could serve them: at that size a
 // step is bound by latency (a few memory round trips), not by arithmetic.

@@ -26,7 +26,7 @@
 //
 // Two forms.  The staged form (dense layers with groups = 1, and depthwise
 // layers, when a pixel's channels are a multiple of 16 bytes and at most 256)
-// gives each CTA one slice of SW output channels of a tile (depthwise: all
+// gives each CTA one slice of 16 or 32 output channels of a tile (depthwise: all
 // channels) and moves its data with asynchronous copies: the slice's weights
 // with one bulk copy issued before the dependency wait (they are constant
 // state), the x_t and x_{t-1} footprints as two TMA boxes right after it
@@ -35,6 +35,8 @@
 // z).  The contraction is split over k when the open locations are too few
 // to occupy the CTA.  The general form loads with plain per-thread accesses
 // and reads weights from global memory; it serves every other shape.
+#include <algorithm>
+
 #include "sc_internal.h"
 #include "sc_ptx.cuh"
 
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
 
 // ------------------------------------------------------------- staged form
 constexpr int FT = 256;                          // threads per CTA
-constexpr int SW = 32;                           // output channels per CTA (dense layers)
+constexpr int SW_WIDE = 32, SW_NARROW = 16;       // output channels per CTA (dense layers)
 constexpr int FLPI = 2;                          // output locations per work item
 constexpr uint64_t LOCAL_WAIT_NS = 1000000000ull;
 
@@ -341,7 +343,7 @@ struct FastArgs {
     int force;
     int n, H, W, C, Ho, Wo, Co, KH, KW, stride, pad, b, nby, nbx, act;
     int sb, nty, ntx, FH, FW, CP, nsl, K;
-    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_red;   // byte offsets from the aligned base
+    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq;   // byte offsets
     float thr;
 };
 
@@ -383,29 +385,33 @@ __device__ __forceinline__ float2 load_pair(const __nv_bfloat16* p)
 {
     return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
 }
-__device__ __forceinline__ void store_pair(float* p, float a, float b) { *reinterpret_cast<float2*>(p) = make_float2(a, b); }
-__device__ __forceinline__ void store_pair(__nv_bfloat16* p, float a, float b)
-{
-    *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(a, b);
-}
 
-template <typename T, bool DW>
-__global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_constant__ CUtensorMap tm_xt,
+template <typename T, bool DW, int SW>
+__global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_constant__ CUtensorMap tm_xt,
                                                                const __grid_constant__ CUtensorMap tm_xp,
+                                                               const __grid_constant__ CUtensorMap tm_z,
+                                                               const __grid_constant__ CUtensorMap tm_sc,
                                                                const FastArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[2];    // 0: weights, 1: footprints
+    __shared__ __align__(8) uint64_t bars[3];    // 0: weights, 1: footprints, 2: z (and shortcut) tile
     __shared__ int s_open[MAX_TILE_BLOCKS];
+    __shared__ int s_max[MAX_TILE_BLOCKS];      // per gate block: largest support sum (float bits)
     __shared__ int s_nloc;
     uint8_t* base = align_smem_1024(smem_raw);
     const T* Xt = reinterpret_cast<const T*>(base);
     const T* Xp = reinterpret_cast<const T*>(base + a.off_xp);
     const T* Ws = reinterpret_cast<const T*>(base + a.off_w);
-    float* R = reinterpret_cast<float*>(base + a.off_r);     // dense only: [FP][CP] residual
+    float* R = reinterpret_cast<float*>(base + a.off_r);      // dense only: [FP][CP] residual
     float* P = reinterpret_cast<float*>(base + a.off_p);
     int* locs = reinterpret_cast<int*>(base + a.off_loc);
-    float* red = reinterpret_cast<float*>(base + a.off_red); // dense only: k-split partial sums
+    float* red = reinterpret_cast<float*>(base + a.off_scr);  // dense: k-split partial sums (scratch)
+    uint8_t* Dq = base + a.off_dq;                            // per footprint pixel: changed
+    const float* Zs = reinterpret_cast<const float*>(base + a.off_z);   // [span*span][ZW] z of the tile
+    const T* Ss = reinterpret_cast<const T*>(base + a.off_sc);          // [span*span][ZW] shortcut of the tile
+    uint8_t* chgs = base + a.off_chg;                                   // owned pixels' previous change flags
+    constexpr int ZW = DW ? 0 : SW;                                     // channels of the z tile (dense)
+    const int zw = DW ? a.Co : ZW;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     constexpr int NW = FT / 32;
     const int sl = DW ? 0 : (int)(blockIdx.x % a.nsl);
@@ -415,11 +421,15 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
     const int oy0 = ty * span, ox0 = tx * span;
     const int fy0 = oy0 * a.stride - a.pad, fx0 = ox0 * a.stride - a.pad;
     const int FP = a.FH * a.FW;
-    const uint32_t bar_w = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]);
+    const int o_base = DW ? 0 : sl * SW;
+    const bool has_sc = a.sc != nullptr;
+    const uint32_t bar_w = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]), bar_z = smem_u32(&bars[2]);
+    const uint32_t ztx = (uint32_t)(span * span * zw) * (4u + (has_sc ? (uint32_t)sizeof(T) : 0u));
 
     if (tid == 0) {
         mbar_init(bar_w, 1);
         mbar_init(bar_x, 1);
+        mbar_init(bar_z, 1);
         fence_mbar_init();
         // the weights are constant state: fetch them before waiting for the producer of x_t
         mbar_arrive_expect_tx(bar_w, a.wbytes);
@@ -428,133 +438,158 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
         prefetch_tmap(&tm_xp);
         s_nloc = 0;
     }
+    if (tid < MAX_TILE_BLOCKS) s_max[tid] = 0;
     grid_dependency_wait();
     if (tid == 0) {
         mbar_arrive_expect_tx(bar_x, 2u * (uint32_t)FP * (uint32_t)a.C * (uint32_t)sizeof(T));
         tma_load_4d(smem_u32(Xt), &tm_xt, bar_x, 0, fx0, fy0, nn);
         tma_load_4d(smem_u32(Xp), &tm_xp, bar_x, 0, fx0, fy0, nn);
+        if (has_sc) {
+            // with a shortcut every location's y is refreshed: z and the shortcut of the whole tile
+            mbar_arrive_expect_tx(bar_z, ztx);
+            tma_load_4d(smem_u32(Zs), &tm_z, bar_z, o_base, ox0, oy0, nn);
+            tma_load_4d(smem_u32(Ss), &tm_sc, bar_z, o_base, ox0, oy0, nn);
+        }
     }
     grid_launch_dependents();
     if (blockIdx.x == 0 && tid == 0) *a.count_next = 0;
-    __syncthreads();   // barrier initialisation visible before anyone waits on it
+
+    // owned input pixels of this tile (every input pixel has exactly one owner tile) and, for
+    // slice 0, their change flags of the previous step
+    const int own_y0 = min(ty * span * a.stride, a.H);
+    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
+    const int own_x0 = min(tx * span * a.stride, a.W);
+    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
+    const int oww = own_x1 - own_x0, npx = (own_y1 - own_y0) * oww;
+    if (sl == 0)
+        for (int q = tid; q < npx; q += FT)
+            chgs[q] = a.chg_prev[((size_t)nn * a.H + own_y0 + q / oww) * a.W + own_x0 + q % oww];
+    __syncthreads();   // barrier initialisation and the flags visible to every thread
     {
         const bool ok = mbar_wait(bar_x, 0, nullptr, a.err, LOCAL_WAIT_NS);
         if (!__syncthreads_and(ok)) {
             // copies may still be in flight into this CTA's shared memory: wait for them (bounded) first
             mbar_wait(bar_x, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            if (has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             return;
         }
     }
-
-    // owned input pixels of this tile (every input pixel has exactly one owner tile)
-    const int own_y0 = min(ty * span * a.stride, a.H);
-    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
-    const int own_x0 = min(tx * span * a.stride, a.W);
-    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
     T* xn = static_cast<T*>(a.xn);
 
-    // residuals, norms and (slice 0) the commit of owned pixels inside the footprint: G lanes per
-    // pixel, 16-byte chunks (a pixel is CH chunks)
+    // residuals, per-chunk partial norms and change bits: one thread per (footprint pixel, 16-byte chunk)
+    constexpr int EPC = 16 / (int)sizeof(T);
+    const int CH = a.C / EPC;
     {
-        constexpr int EPC = 16 / (int)sizeof(T);
-        const int CH = a.C / EPC;
-        int lg = 0;
-        while ((1 << lg) < CH && lg < 5) ++lg;
-        const int G = 1 << lg, gpw = 32 >> lg, sub = lane & (G - 1);
-        for (int q0 = warp * gpw; q0 < FP; q0 += NW * gpw) {
-            const int q = q0 + (lane >> lg);
-            const bool valid = q < FP;
-            const uint4* xs = reinterpret_cast<const uint4*>(Xt + (size_t)(valid ? q : 0) * a.C);
-            const uint4* ps = reinterpret_cast<const uint4*>(Xp + (size_t)(valid ? q : 0) * a.C);
+        float* Pp = reinterpret_cast<float*>(base + a.off_scr);            // [FP][CH]
+        uint8_t* Dp = base + a.off_scr + (size_t)FP * CH * sizeof(float);   // [FP][CH]
+        for (int it = tid; it < FP * CH; it += FT) {
+            const int q = it / CH, k = it - (it / CH) * CH;
+            const uint4 av = reinterpret_cast<const uint4*>(Xt + (size_t)q * a.C)[k];
+            const uint4 bv = reinterpret_cast<const uint4*>(Xp + (size_t)q * a.C)[k];
+            float r[8];
+            const int ne = chunk_residual(av, bv, r, (T*)nullptr);
             float sum = 0.f;
-            unsigned d = 0;
-            if (valid) {
-                for (int k = sub; k < CH; k += G) {
-                    const uint4 av = xs[k], bv = ps[k];
-                    float r[8];
-                    const int ne = chunk_residual(av, bv, r, (T*)nullptr);
 #pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        if (e < ne) sum += fabsf(r[e]);
-                    d |= (av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w);
-                    if (!DW) {
-                        float4* rr = reinterpret_cast<float4*>(R + (size_t)q * a.CP + k * EPC);
-                        rr[0] = make_float4(r[0], r[1], r[2], r[3]);
-                        if (EPC == 8) rr[1] = make_float4(r[4], r[5], r[6], r[7]);
-                    }
-                }
-            }
-            for (int off = 1; off < G; off <<= 1) {
-                sum += __shfl_xor_sync(0xffffffffu, sum, off);
-                d |= __shfl_xor_sync(0xffffffffu, d, off);
-            }
-            if (valid && sub == 0) P[q] = sum;
-            if (sl == 0 && valid) {
-                const int iy = fy0 + q / a.FW, ix = fx0 + q % a.FW;
-                if (iy >= own_y0 && iy < own_y1 && ix >= own_x0 && ix < own_x1) {
-                    const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
-                    if (d || a.chg_prev[pix]) {
-                        uint4* dst = reinterpret_cast<uint4*>(xn) + pix * CH;
-                        for (int k = sub; k < CH; k += G) dst[k] = xs[k];
-                    }
-                    if (sub == 0) a.chg_cur[pix] = d ? 1 : 0;
-                }
+            for (int e = 0; e < 8; ++e)
+                if (e < ne) sum += fabsf(r[e]);
+            Pp[it] = sum;
+            Dp[it] = ((av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w)) != 0u;
+            if (!DW) {
+                float4* rr = reinterpret_cast<float4*>(R + (size_t)q * a.CP + k * EPC);
+                rr[0] = make_float4(r[0], r[1], r[2], r[3]);
+                if (EPC == 8) rr[1] = make_float4(r[4], r[5], r[6], r[7]);
             }
         }
+        __syncthreads();
+        // per pixel: the l1 norm (chunk partials in channel order) and whether any bit changed
+        for (int q = tid; q < FP; q += FT) {
+            float sum = 0.f;
+            unsigned d = 0;
+            for (int k = 0; k < CH; ++k) {
+                sum += Pp[q * CH + k];
+                d |= Dp[q * CH + k];
+            }
+            P[q] = sum;
+            Dq[q] = (uint8_t)d;
+        }
     }
-    // owned pixels outside the footprint (input rows or columns no output location reads)
+    __syncthreads();
+
+    // slice 0: the commit of x_t for the owned pixels (one thread per pixel and chunk inside the
+    // footprint, a warp per pixel outside it), and the pixels' change flags
     if (sl == 0) {
+        for (int it = tid; it < npx * CH; it += FT) {
+            const int q = it / CH, k = it - (it / CH) * CH;
+            const int iy = own_y0 + q / oww, ix = own_x0 + q % oww;
+            const int fy = iy - fy0, fx = ix - fx0;
+            if (fy >= a.FH || fx >= a.FW) continue;
+            const int fq = fy * a.FW + fx;
+            const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
+            const bool changed = Dq[fq] != 0;
+            if (changed || chgs[q])
+                (reinterpret_cast<uint4*>(xn) + pix * CH)[k] = reinterpret_cast<const uint4*>(Xt + (size_t)fq * a.C)[k];
+            if (k == 0) a.chg_cur[pix] = changed ? 1 : 0;
+        }
         const T* xt = static_cast<const T*>(a.xt);
         const T* xp = static_cast<const T*>(a.xp);
-        const int ow = own_x1 - own_x0, npx = (own_y1 - own_y0) * ow;
         for (int q = warp; q < npx; q += NW) {
-            const int iy = own_y0 + q / ow, ix = own_x0 + q % ow;
+            const int iy = own_y0 + q / oww, ix = own_x0 + q % oww;
             if (iy - fy0 < a.FH && ix - fx0 < a.FW) continue;   // done from the footprint
             const size_t pix = ((size_t)nn * a.H + iy) * a.W + ix;
             unsigned d = 0;
             for (int c = lane; c < a.C; c += 32) d |= bits_of(xt[pix * a.C + c]) ^ bits_of(xp[pix * a.C + c]);
             const bool changed = __any_sync(0xffffffffu, d != 0);
-            if (changed || a.chg_prev[pix])
+            if (changed || chgs[q])
                 for (int c = lane; c < a.C; c += 32) xn[pix * a.C + c] = xt[pix * a.C + c];
             if (lane == 0) a.chg_cur[pix] = changed ? 1 : 0;
         }
     }
-    __syncthreads();
 
-    // block gates of the tile (a warp per gate block)
-    for (int bq = warp; bq < a.sb * a.sb; bq += NW) {
-        const int bi = bq / a.sb, bj = bq - (bq / a.sb) * a.sb;
-        const int by = ty * a.sb + bi, bx = tx * a.sb + bj;
-        int open = 0;
-        if (by < a.nby && bx < a.nbx) {
-            const int bh = min(a.b, a.Ho - by * a.b), bw = min(a.b, a.Wo - bx * a.b);
-            float best = -1.f;
-            for (int q = lane; q < bh * bw; q += 32) {
-                const int li = bi * a.b + q / bw, lj = bj * a.b + q % bw;
-                float S = 0.f;
-                for (int kh = 0; kh < a.KH; ++kh)
-                    for (int kw = 0; kw < a.KW; ++kw) S += P[(li * a.stride + kh) * a.FW + lj * a.stride + kw];
-                best = fmaxf(best, S);
-            }
-            best = warp_max(best);
-            open = (a.force || best > a.thr) ? 1 : 0;
-            if (sl == 0 && lane == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
+    // block gates: per output location its support sum, per block the maximum (the sums are
+    // non-negative, so their float bits order like integers)
+    for (int q = tid; q < span * span; q += FT) {
+        const int li = q / span, lj = q - (q / span) * span;
+        if (oy0 + li >= a.Ho || ox0 + lj >= a.Wo) continue;
+        const float* Pl = P + li * a.stride * a.FW + lj * a.stride;
+        float S = 0.f;
+        if (a.KH == 3 && a.KW == 3) {   // the same order, with the nine loads issued together
+            float v[9];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) v[t] = Pl[(t / 3) * a.FW + t % 3];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) S += v[t];
+        } else {
+            for (int kh = 0; kh < a.KH; ++kh)
+                for (int kw = 0; kw < a.KW; ++kw) S += Pl[kh * a.FW + kw];
         }
-        if (lane == 0) s_open[bq] = open;
+        atomicMax(&s_max[(li / a.b) * a.sb + lj / a.b], __float_as_int(S));
     }
     __syncthreads();
-    if (sl == 0 && warp == 0) {
-        const int nb = a.sb * a.sb;
-        const int o = lane < nb ? s_open[lane] : 0;
-        const unsigned bal = __ballot_sync(0xffffffffu, o);
-        int basei = 0;
-        if (lane == 0 && bal) basei = atomicAdd(a.count_cur, __popc(bal));
-        basei = __shfl_sync(0xffffffffu, basei, 0);
-        if (o) {
-            const int by = ty * a.sb + lane / a.sb, bx = tx * a.sb + lane % a.sb;
-            a.list[basei + __popc(bal & ((1u << lane) - 1u))] = (int32_t)(((size_t)nn * a.nby + by) * a.nbx + bx);
+    if (tid < a.sb * a.sb) {
+        const int by = ty * a.sb + tid / a.sb, bx = tx * a.sb + tid % a.sb;
+        int open = 0;
+        if (by < a.nby && bx < a.nbx) {
+            open = (a.force || __int_as_float(s_max[tid]) > a.thr) ? 1 : 0;
+            if (sl == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
         }
+        s_open[tid] = open;
+    }
+    __syncthreads();
+    bool any_open = false;
+    for (int bq = 0; bq < a.sb * a.sb; ++bq) any_open |= s_open[bq] != 0;
+    if (tid == 0 && any_open && !has_sc) {
+        // the z tile of a tile with open blocks (without a shortcut only those are touched)
+        mbar_arrive_expect_tx(bar_z, ztx);
+        tma_load_4d(smem_u32(Zs), &tm_z, bar_z, o_base, ox0, oy0, nn);
+    }
+    // the open blocks into the list: the slot comes back while the convolution runs
+    int list_base = 0, list_open = 0;
+    unsigned list_bal = 0;
+    if (sl == 0 && warp == 0) {
+        list_open = lane < a.sb * a.sb ? s_open[lane] : 0;
+        list_bal = __ballot_sync(0xffffffffu, list_open);
+        if (lane == 0 && list_bal) list_base = atomicAdd(a.count_cur, __popc(list_bal));
     }
     for (int q = tid; q < span * span; q += FT) {
         const int li = q / span, lj = q - (q / span) * span;
@@ -562,16 +597,20 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
             locs[atomicAdd(&s_nloc, 1)] = (li << 16) | lj;
     }
     {
-        const bool ok = mbar_wait(bar_w, 0, nullptr, a.err, LOCAL_WAIT_NS);
+        bool ok = mbar_wait(bar_w, 0, nullptr, a.err, LOCAL_WAIT_NS);
+        if (any_open || has_sc) ok = ok && mbar_wait(bar_z, 0, nullptr, a.err, LOCAL_WAIT_NS);
         if (!__syncthreads_and(ok)) {
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            if (any_open || has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             return;
         }
     }
 
     const int M = s_nloc;
     T* y = static_cast<T*>(a.y);
-    const bool y_here = y != nullptr && a.sc == nullptr;
+    auto y_of = [&](float zv, int zi) {   // the layer output at tile element zi (location * zw + channel)
+        return from_f32<T>(activate(has_sc ? zv + to_f32(Ss[zi]) : zv, a.act));
+    };
     if (DW) {
         // a thread per channel pair (weights in registers) and a share of the open locations
         const int NCP = a.C / 2, ngrp = FT / NCP;
@@ -584,8 +623,6 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
             for (int m = g; m < M; m += ngrp) {
                 const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
                 const int p0 = li * a.stride * a.FW + lj * a.stride;
-                const size_t zo = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + c;
-                const float2 zold = *reinterpret_cast<const float2*>(a.z + zo);
                 float acc0 = 0.f, acc1 = 0.f;
                 if (a.KH == 3 && a.KW == 3) {
 #pragma unroll
@@ -607,21 +644,23 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
                             acc1 = fmaf(w.y, xa.y - xb.y, acc1);
                         }
                 }
-                const float z0 = zold.x + acc0, z1 = zold.y + acc1;
+                const int zi = (li * span + lj) * zw + c;
+                const float z0 = Zs[zi] + acc0, z1 = Zs[zi + 1] + acc1;
+                const size_t zo = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + c;
                 *reinterpret_cast<float2*>(a.z + zo) = make_float2(z0, z1);
-                if (y_here) store_pair(y + zo, activate(z0, a.act), activate(z1, a.act));
+                if (y) {
+                    const T y0 = y_of(z0, zi), y1 = y_of(z1, zi + 1);
+                    y[zo] = y0;
+                    y[zo + 1] = y1;
+                }
             }
         }
     } else {
         constexpr int NQ = SW / 4;
         const int items = (M + FLPI - 1) / FLPI * NQ;
         const int parts = items == 0 ? 1 : max(1, min(8, FT / items));
-        const int o_base = sl * SW;
-        // pre: also load the item's z values now, so that their latency hides behind the contraction
-        auto contract = [&](int item, int k_lo, int k_hi, float (&acc)[FLPI][4], long long (&zl)[FLPI],
-                            float (&zv)[FLPI][4], bool pre) {
+        auto contract = [&](int item, int k_lo, int k_hi, float (&acc)[FLPI][4], int (&lz)[FLPI]) {
             const int q = item % NQ, mi = item / NQ;
-            const int o = o_base + q * 4;
             int rb[FLPI];
 #pragma unroll
             for (int u = 0; u < FLPI; ++u) {
@@ -629,16 +668,13 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
                 if (m < M) {
                     const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
                     rb[u] = (li * a.stride * a.FW + lj * a.stride) * a.CP;
-                    zl[u] = ((long long)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj;
+                    lz[u] = li * span + lj;
                 } else {
                     rb[u] = 0;
-                    zl[u] = -1;
+                    lz[u] = -1;
                 }
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    acc[u][j] = 0.f;
-                    zv[u][j] = (pre && zl[u] >= 0 && o + j < a.Co) ? a.z[(size_t)zl[u] * a.Co + o + j] : 0.f;
-                }
+                for (int j = 0; j < 4; ++j) acc[u][j] = 0.f;
             }
             // k = tap * C + ci; walk the taps of [k_lo, k_hi)
             int tap = k_lo / a.C, ci = k_lo - tap * a.C;
@@ -665,37 +701,39 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
                 ++tap;
             }
         };
-        auto store = [&](int item, const float (&acc)[FLPI][4], const long long (&zl)[FLPI],
-                         const float (&zv)[FLPI][4]) {
-            const int o = o_base + (item % NQ) * 4;
+        auto store = [&](int item, const float (&acc)[FLPI][4], const int (&lz)[FLPI]) {
+            const int oq = (item % NQ) * 4;
 #pragma unroll
             for (int u = 0; u < FLPI; ++u) {
-                if (zl[u] < 0) continue;
+                if (lz[u] < 0) continue;
+                const int li = lz[u] / span, lj = lz[u] - (lz[u] / span) * span;
+                const size_t zrow = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co;
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
-                    if (o + j >= a.Co) continue;
-                    const size_t zo = (size_t)zl[u] * a.Co + o + j;
-                    const float znew = zv[u][j] + acc[u][j];
-                    a.z[zo] = znew;
-                    if (y_here) y[zo] = from_f32<T>(activate(znew, a.act));
+                    const int o = o_base + oq + j;
+                    if (o >= a.Co) continue;
+                    const int zi = lz[u] * ZW + oq + j;
+                    const float znew = Zs[zi] + acc[u][j];
+                    a.z[zrow + o] = znew;
+                    if (y) y[zrow + o] = y_of(znew, zi);
                 }
             }
         };
         if (parts == 1) {
             for (int it = tid; it < items; it += FT) {
-                float acc[FLPI][4], zv[FLPI][4];
-                long long zl[FLPI];
-                contract(it, 0, a.K, acc, zl, zv, true);
-                store(it, acc, zl, zv);
+                float acc[FLPI][4];
+                int lz[FLPI];
+                contract(it, 0, a.K, acc, lz);
+                store(it, acc, lz);
             }
         } else {
             // too few open locations to occupy the CTA: split k over `parts` thread groups
             const int item = tid % items, part = tid / items;
-            float acc[FLPI][4], zv[FLPI][4];
-            long long zl[FLPI];
+            float acc[FLPI][4];
+            int lz[FLPI];
             if (part < parts) {
                 const int k_lo = (int)((long long)a.K * part / parts), k_hi = (int)((long long)a.K * (part + 1) / parts);
-                contract(item, k_lo, k_hi, acc, zl, zv, part == 0);
+                contract(item, k_lo, k_hi, acc, lz);
                 if (part > 0) {
 #pragma unroll
                     for (int u = 0; u < FLPI; ++u)
@@ -710,40 +748,48 @@ __global__ void __launch_bounds__(FT) step_local_staged_kernel(const __grid_cons
                     for (int u = 0; u < FLPI; ++u)
 #pragma unroll
                         for (int j = 0; j < 4; ++j) acc[u][j] += red[((pp - 1) * items + item) * (FLPI * 4) + u * 4 + j];
-                store(item, acc, zl, zv);
+                store(item, acc, lz);
             }
         }
     }
 
-    if (y != nullptr && a.sc != nullptr) {
-        __syncthreads();
-        const T* sc = static_cast<const T*>(a.sc);
+    // with a shortcut: y = act(z + shortcut) at the tile's closed locations (the open ones got theirs above)
+    if (y != nullptr && has_sc) {
         const int th = min(span, a.Ho - oy0), tw = min(span, a.Wo - ox0);
-        const int c0 = DW ? 0 : sl * SW, nc = DW ? a.Co : min(SW, a.Co - sl * SW);
+        const int nc = DW ? a.Co : min(SW, a.Co - o_base);
         for (int it = tid; it < th * tw * nc; it += FT) {
-            const int c = c0 + it % nc, p = it / nc;
-            const size_t zo = (((size_t)nn * a.Ho + oy0 + p / tw) * a.Wo + ox0 + p % tw) * a.Co + c;
-            y[zo] = from_f32<T>(activate(a.z[zo] + to_f32(sc[zo]), a.act));
+            const int c = it % nc, p = it / nc;
+            const int li = p / tw, lj = p - (p / tw) * tw;
+            if (s_open[(li / a.b) * a.sb + lj / a.b]) continue;
+            const int zi = (li * span + lj) * zw + c;
+            y[(((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + o_base + c] = y_of(Zs[zi], zi);
+        }
+    }
+    if (sl == 0 && warp == 0 && list_bal) {
+        const int basei = __shfl_sync(0xffffffffu, list_base, 0);
+        if (list_open) {
+            const int by = ty * a.sb + lane / a.sb, bx = tx * a.sb + lane % a.sb;
+            a.list[basei + __popc(list_bal & ((1u << lane) - 1u))] = (int32_t)(((size_t)nn * a.nby + by) * a.nbx + bx);
         }
     }
 }
 
-// Weights of the staged form, in the layer's dtype: dense [slice][K][SW]
+// Weights of the staged form, in the layer's dtype: dense [slice][K][sw]
 // (K index = tap * c_in + ci, channels past c_out zero), depthwise [taps][C].
 template <typename T>
 __global__ void pack_local_weights_kernel(const float* __restrict__ wcc, T* __restrict__ out, int K, int Co,
-                                          int nsl, int dw)
+                                          int nsl, int sw, int dw)
 {
-    const long long total = dw ? (long long)K * Co : (long long)nsl * K * SW;
+    const long long total = dw ? (long long)K * Co : (long long)nsl * K * sw;
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         if (dw) {
             out[i] = from_f32<T>(wcc[i]);
         } else {
-            const int j = (int)(i % SW);
-            const long long rest = i / SW;
+            const int j = (int)(i % sw);
+            const long long rest = i / sw;
             const int k = (int)(rest % K), sl = (int)(rest / K);
-            const int o = sl * SW + j;
+            const int o = sl * sw + j;
             out[i] = from_f32<T>(o < Co ? wcc[(size_t)k * Co + o] : 0.f);
         }
     }
@@ -791,9 +837,12 @@ const void* kernel_of(const Layer& L)
 // ------------------------------------------------------ staged form, host side
 struct StagedShape {
     LocalShape g;
+    int sw;          // output channels per CTA (dense layers)
     int nsl;
+    int zw;          // channels of the z / shortcut tile boxes
+    size_t own_max;  // most input pixels a tile owns
     uint32_t wbytes;
-    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_red;
+    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq;
     size_t smem;
 };
 
@@ -809,31 +858,50 @@ StagedShape staged_shape(const Layer& L, int sb)
     const bool dw = is_depthwise(L);
     const size_t fp = (size_t)t.g.FH * t.g.FW;
     const int K = L.p.k_h * L.p.k_w * L.p.c_in;
-    t.nsl = dw ? 1 : (L.p.c_out + SW - 1) / SW;
-    const size_t wb = dw ? (size_t)L.p.k_h * L.p.k_w * L.p.c_in * L.esize : (size_t)K * SW * L.esize;
+    // small tiles with few output channels: narrower slices spread an open tile over more SMs
+    t.sw = (t.g.span <= 4 && L.p.c_out <= 32) ? SW_NARROW : SW_WIDE;
+    t.nsl = dw ? 1 : (L.p.c_out + t.sw - 1) / t.sw;
+    t.zw = dw ? L.p.c_out : t.sw;
+    const size_t wb = dw ? (size_t)L.p.k_h * L.p.k_w * L.p.c_in * L.esize : (size_t)K * t.sw * L.esize;
     t.wbytes = (uint32_t)((wb + 15) & ~(size_t)15);
+    // largest owned input region of a tile (the last tile row / column owns the rest of the frame)
+    const int span_in = t.g.span * L.p.stride;
+    const int nty = (L.nby + sb - 1) / sb, ntx = (L.nbx + sb - 1) / sb;
+    const int own_h = std::max(std::min(span_in, L.p.h), L.p.h - (nty - 1) * span_in);
+    const int own_w = std::max(std::min(span_in, L.p.w), L.p.w - (ntx - 1) * span_in);
+    t.own_max = (size_t)std::max(own_h, 0) * std::max(own_w, 0);
+    const size_t tile_elems = (size_t)t.g.span * t.g.span * t.zw;
     const uint32_t xb = up128(fp * L.p.c_in * L.esize);
     t.off_xp = xb;
     t.off_w = 2 * xb;
     t.off_r = t.off_w + up128(t.wbytes);
     t.off_p = t.off_r + (dw ? 0 : up128(fp * t.g.CP * sizeof(float)));
     t.off_loc = t.off_p + up128(fp * sizeof(float));
-    t.off_red = t.off_loc + up128((size_t)t.g.span * t.g.span * sizeof(int));
-    t.smem = (size_t)t.off_red + (dw ? 0 : up128((size_t)FT * FLPI * 4 * sizeof(float))) + 1024;
+    t.off_scr = t.off_loc + up128((size_t)t.g.span * t.g.span * sizeof(int));
+    // scratch: the footprint pass's chunk partials, later (dense) the k-split partial sums
+    const size_t chunks = fp * (L.p.c_in * L.esize / 16);
+    const size_t scr = std::max(chunks * (sizeof(float) + 1), dw ? (size_t)0 : (size_t)FT * FLPI * 4 * sizeof(float));
+    t.off_z = t.off_scr + up128(scr);
+    t.off_sc = t.off_z + up128(tile_elems * sizeof(float));
+    t.off_chg = t.off_sc + (L.p.emit_y ? up128(tile_elems * L.esize) : 0);
+    t.off_dq = t.off_chg + up128(t.own_max);
+    t.smem = (size_t)t.off_dq + up128(fp) + 1024;
     return t;
 }
 
 // The staged form needs TMA boxes of the footprint (a pixel's channels a
-// multiple of 16 bytes, every box edge at most 256) and a dense (groups = 1)
-// or depthwise layer.
+// multiple of 16 bytes, every box edge at most 256), of the z tile (c_out a
+// multiple of 4) and of the shortcut tile (c_out a multiple of 16 bytes of
+// the dtype), and a dense (groups = 1) or depthwise layer.
 bool staged_ok(const Layer& L, StagedShape* out)
 {
     if (!(L.p.groups == 1 || is_depthwise(L))) return false;
     if ((L.p.c_in * L.esize) % 16 || L.p.c_in > 256) return false;
+    if (L.p.c_out % 4 || (L.p.emit_y && (L.p.c_out * L.esize) % 16)) return false;
     int sb = L.p.block >= 4 ? 1 : (4 + L.p.block - 1) / L.p.block;
     StagedShape t = staged_shape(L, sb);
     while (t.smem > LOCAL_MAX_SMEM && sb > 1) t = staged_shape(L, --sb);
-    if (t.smem > LOCAL_MAX_SMEM || t.g.FH > 256 || t.g.FW > 256) return false;
+    if (t.smem > LOCAL_MAX_SMEM || t.g.FH > 256 || t.g.FW > 256 || t.g.span > 256 || t.zw > 256) return false;
     if ((long long)L.p.n_streams * ((L.nby + sb - 1) / sb) * ((L.nbx + sb - 1) / sb) * t.nsl > 0x7fffffffLL)
         return false;
     if (out) *out = t;
@@ -856,13 +924,34 @@ bool encode_footprint_map(CUtensorMap* m, const void* base, const Layer& L, cons
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-const void* staged_kernel_of(const Layer& L)
+// Tile boxes of an output-shaped tensor [n][ho][wo][c_out]: z (fp32) or the shortcut (dtype).
+bool encode_tile_map(CUtensorMap* m, const void* base, const Layer& L, const StagedShape& t, bool fp32)
 {
-    const bool dw = is_depthwise(L);
-    if (L.p.dtype == SKIPCONV_BF16)
-        return dw ? (const void*)step_local_staged_kernel<__nv_bfloat16, true>
-                  : (const void*)step_local_staged_kernel<__nv_bfloat16, false>;
-    return dw ? (const void*)step_local_staged_kernel<float, true> : (const void*)step_local_staged_kernel<float, false>;
+    EncodeTiledFn enc = encode_tiled_fn();
+    if (!enc) return false;
+    const cuuint64_t Co = L.p.c_out, Wo = L.wo, Ho = L.ho, N = L.p.n_streams, es = fp32 ? 4 : L.esize;
+    cuuint64_t dims[4] = {Co, Wo, Ho, N};
+    cuuint64_t strides[3] = {Co * es, Wo * Co * es, Ho * Wo * Co * es};
+    cuuint32_t box[4] = {(cuuint32_t)t.zw, (cuuint32_t)t.g.span, (cuuint32_t)t.g.span, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUtensorMapDataType dt = fp32 || L.p.dtype != SKIPCONV_BF16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                                                     : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return enc(m, dt, 4, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <typename T>
+const void* staged_kernel_of(const Layer& L, int sw)
+{
+    if (is_depthwise(L)) return (const void*)step_local_staged_kernel<T, true, SW_WIDE>;
+    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<T, false, SW_NARROW>
+                           : (const void*)step_local_staged_kernel<T, false, SW_WIDE>;
+}
+
+const void* staged_kernel_of(const Layer& L, int sw)
+{
+    return L.p.dtype == SKIPCONV_BF16 ? staged_kernel_of<__nv_bfloat16>(L, sw) : staged_kernel_of<float>(L, sw);
 }
 
 cudaLaunchConfig_t pdl_config(const Layer& L, long long grid, int threads, size_t smem, cudaLaunchAttribute* attr)
@@ -899,8 +988,9 @@ cudaError_t step_local_prepare(Layer& L)
 {
     StagedShape t;
     if (staged_ok(L, &t)) {
-        if (!encode_footprint_map(&L.tmap_fp[0], L.xbuf[0], L, t) || !encode_footprint_map(&L.tmap_fp[1], L.xbuf[1], L, t)) {
-            set_error("tensor map of the state frames rejected");
+        if (!encode_footprint_map(&L.tmap_fp[0], L.xbuf[0], L, t) || !encode_footprint_map(&L.tmap_fp[1], L.xbuf[1], L, t) ||
+            !encode_tile_map(&L.tmap_ztile, L.z, L, t, true)) {
+            set_error("tensor map of the layer state rejected");
             return cudaErrorInvalidValue;
         }
         const size_t bytes = (size_t)t.wbytes * t.nsl;
@@ -914,19 +1004,19 @@ cudaError_t step_local_prepare(Layer& L)
         if (e != cudaSuccess) return e;
         const bool dw = is_depthwise(L);
         const int K = L.p.k_h * L.p.k_w * L.p.c_in;
-        const long long total = dw ? (long long)K * L.p.c_out : (long long)t.nsl * K * SW;
+        const long long total = dw ? (long long)K * L.p.c_out : (long long)t.nsl * K * t.sw;
         const int grid = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
         if (L.p.dtype == SKIPCONV_BF16)
             pack_local_weights_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(
-                L.w_cc, (__nv_bfloat16*)L.w_loc, dw ? L.p.k_h * L.p.k_w : K, L.p.c_out, t.nsl, dw ? 1 : 0);
+                L.w_cc, (__nv_bfloat16*)L.w_loc, dw ? L.p.k_h * L.p.k_w : K, L.p.c_out, t.nsl, t.sw, dw ? 1 : 0);
         else
             pack_local_weights_kernel<float><<<grid, 256, 0, L.stream>>>(L.w_cc, (float*)L.w_loc,
                                                                          dw ? L.p.k_h * L.p.k_w : K, L.p.c_out,
-                                                                         t.nsl, dw ? 1 : 0);
+                                                                         t.nsl, t.sw, dw ? 1 : 0);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         L.local_staged = 1;
-        return ensure_dynamic_smem(staged_kernel_of(L), t.smem);
+        return ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
     }
     L.local_staged = 0;
     return ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
@@ -969,13 +1059,19 @@ cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* short
         a.ntx = (L.nbx + t.g.sb - 1) / t.g.sb;
         a.FH = t.g.FH; a.FW = t.g.FW; a.CP = t.g.CP; a.nsl = t.nsl; a.K = L.p.k_h * L.p.k_w * L.p.c_in;
         a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
-        a.off_red = t.off_red;
+        a.off_scr = t.off_scr; a.off_z = t.off_z; a.off_sc = t.off_sc; a.off_chg = t.off_chg; a.off_dq = t.off_dq;
         a.thr = L.gate_thr;
+        alignas(64) CUtensorMap tm_sc = L.tmap_ztile;   // unused without a shortcut
+        if (a.sc && !encode_tile_map(&tm_sc, a.sc, L, t, false)) {
+            set_error("tensor map of the shortcut rejected");
+            return cudaErrorInvalidValue;
+        }
         const long long grid = (long long)a.n * a.nty * a.ntx * t.nsl;
         cudaLaunchConfig_t cfg = pdl_config(L, grid, FT, t.smem, attr);
         const CUtensorMap* tm_xp = &L.tmap_fp[cur];
-        void* args[] = {&tm_xt, const_cast<CUtensorMap*>(tm_xp), &a};
-        return cudaLaunchKernelExC(&cfg, staged_kernel_of(L), args);
+        CUtensorMap* tm_z = const_cast<CUtensorMap*>(&L.tmap_ztile);
+        void* args[] = {&tm_xt, const_cast<CUtensorMap*>(tm_xp), tm_z, &tm_sc, &a};
+        return cudaLaunchKernelExC(&cfg, staged_kernel_of(L, t.sw), args);
     }
     const LocalShape s = choose_shape(L);
     LocalArgs a;
