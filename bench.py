@@ -58,6 +58,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the single-layer and stacked workloads (c0-c3)")
+    ap.add_argument("--link", choices=("both", "on", "off"), default="both",
+                    help="stack propagation for the stacked workloads: also time linked stacks (both), "
+                         "link them throughout (on), or not at all (off)")
     ap.add_argument("--workloads-only", default=None, metavar="NAMES",
                     help="run only these of the single-layer and stacked workloads (comma-separated, e.g. c2,c3) "
                          "and print their report; for profiling them")
@@ -340,15 +343,34 @@ def layer_roof(L, n, h, w, ho, wo, esz, locs, chg, emit_y, conv_path, tc_peak, h
     return flops, bytes_, max(flops / (peak * 1e12), bytes_ / (hbm * 1e9))
 
 
-def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c2", "c3")):
-    """The single-layer (c0, c1) and stacked (c2 pose-like, c3 MBConv-like)
-    workloads, run free: each layer steps on the previous layer's y (and its
+def link_stack(wl, lays):
+    """Stack propagation: link each layer to the layers whose y it takes as
+    x_t and as the shortcut (the frame input and external shortcuts stay
+    unlinked; layers that cannot take links keep reading whole frames)."""
+    from paper_2104_11487_gb300._lib import SkipConvError
+    linked = 0
+    for li, L in enumerate(wl.layers):
+        if li == 0:
+            continue
+        try:
+            lays[li].link(lays[li - 1], None if L.shortcut <= 0 else lays[L.shortcut - 1])
+            linked += 1
+        except SkipConvError:
+            pass
+    return linked
+
+
+def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c2", "c3", "dw3"), link="both"):
+    """The single-layer (c0, c1) and stacked (c2 pose-like, c3 MBConv-like,
+    dw3 a frame-sized depthwise stack for stack propagation) workloads, run free: each layer steps on the previous layer's y (and its
     shortcut) on the device, one frame after the other, with an L2 flush
     between frames.  Frame 0 is the key frame; `warmup` frames follow
     untimed; the rest of the video is timed with CUDA events around each
     frame.  A second pass with the library's per-launch events gives each
     layer's kernel time, and a third (host-synchronised) pass counts each
-    layer's open locations and changed input pixels for its roofline."""
+    layer's open locations and changed input pixels for its roofline.
+    link: "both" adds a fourth pass with the stack's layers linked (stack
+    propagation, identical results); "on" links them for every pass."""
     import synth
     from paper_2104_11487_gb300 import (SkipConvLayer, device_tensor, skipconv_get_y, skipconv_profile,
                                         skipconv_profile_read)
@@ -357,7 +379,9 @@ def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c
         wl = synth.make_workload(name)
         dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
         esz = 2 if wl.dtype == "bf16" else 4
-        frames = [torch.from_numpy(np.ascontiguousarray(wl.frames[t])).cuda().to(dt) for t in range(wl.T)]
+        # (a generated video may reuse one buffer for every frame: copy each frame as it comes)
+        src = (wl.frames[t] for t in range(wl.T)) if isinstance(wl.frames, np.ndarray) else (f for _, f in wl.frames)
+        frames = [torch.from_numpy(np.ascontiguousarray(f)).cuda().to(dt) for f in src]
         stacked = len(wl.layers) > 1
         lays, ys, dims = [], [], []
         h, w = wl.h, wl.w
@@ -371,6 +395,7 @@ def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c
             dims.append((h, w, lay.info.ho, lay.info.wo))
             h, w = lay.info.ho, lay.info.wo
         stream = lays[0].stream
+        n_links = link_stack(wl, lays) if (stacked and link == "on") else 0
 
         def frame_step(x):
             stack = [x]
@@ -447,7 +472,25 @@ def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c
         t_frame = statistics.median(ms) * 1e-3
         report[name] = {"frames": len(timed), "dtype": wl.dtype, "ms_per_frame": t_frame * 1e3,
                         "frames_per_s": wl.n / t_frame, "eff_tflops": flops_sum / t_frame / 1e12,
-                        "stack_roofline_frac": t_roof_sum / t_frame, "layers": per_layer}
+                        "stack_roofline_frac": t_roof_sum / t_frame, "layers": per_layer,
+                        "linked_layers": n_links}
+        if stacked and link == "both":
+            # 4) the same frames with stack propagation (each layer linked to its producers)
+            n_links = link_stack(wl, lays)
+            reset()
+            for t in range(warmup + 1):
+                frame_step(frames[t])
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in timed]
+            torch.cuda.synchronize()
+            for i, t in enumerate(timed):
+                flush_l2(flush)
+                ev[i][0].record(stream)
+                frame_step(frames[t])
+                ev[i][1].record(stream)
+            torch.cuda.synchronize()
+            t_link = statistics.median([a.elapsed_time(b) for a, b in ev]) * 1e-3
+            report[name]["propagation"] = {"linked_layers": n_links, "ms_per_frame": t_link * 1e3,
+                                           "frames_per_s": wl.n / t_link}
         for lay in lays:
             lay.close()
         del frames
@@ -556,7 +599,8 @@ def main():
 
     if args.workloads_only:
         flush = None if args.no_flush else torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-        rep = workloads_report(torch, flush, tc_peak, hbm, names=tuple(args.workloads_only.split(",")))
+        rep = workloads_report(torch, flush, tc_peak, hbm, names=tuple(args.workloads_only.split(",")),
+                               link=args.link)
         if rank == 0:
             print(json.dumps({"other_workloads": rep}), flush=True)
         ranks.close()
@@ -686,7 +730,7 @@ def main():
 
     # 5) the single-layer and stacked workloads
     if not args.no_workloads:
-        line["other_workloads"] = workloads_report(torch, flush, tc_peak, hbm)
+        line["other_workloads"] = workloads_report(torch, flush, tc_peak, hbm, link=args.link)
 
     # 6) the CPU oracle on the host cores (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -140,6 +140,27 @@ SKIPCONV_API int skipconv_reset_state(skipconv_handle h);
  * x_t and shortcut must stay valid until the stream reaches this work. */
 SKIPCONV_API int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut);
 
+/* Stack propagation: the input of layer l+1 changes only where layer l's
+ * output changed (the residual of Eq. 2 is zero elsewhere).  Declares that
+ * this layer's x_t is producer_x's y and, if producer_sc is not NULL, that
+ * its shortcut is producer_sc's y.  Every layer that keeps y publishes, per
+ * gate block, whether its last step may have changed y (an open block, or a
+ * changed shortcut).  At a step whose x_t (and shortcut) are those producers'
+ * y and whose producers each stepped exactly once since this layer last did,
+ * a tile whose footprint saw no such change, that committed no change at the
+ * previous step and whose shortcut did not change, skips reading its inputs:
+ * its residual is zero there, so the full step would keep every block closed
+ * and write nothing.  Results are identical to unlinked steps.  Otherwise
+ * (another x_t, a producer that stepped twice or not at all, key frames) the
+ * step reads the whole frame as usual.  producer_x = NULL removes the links.
+ * Errors: INVALID (NULL handle, self link, shortcut link without x link,
+ * shapes, dtypes or streams that do not match), UNSUPPORTED (this layer not on
+ * the one-launch CUDA-core step with TMA footprints, or a producer that keeps
+ * no y or is not on the one-launch CUDA-core step).  Destroying a producer
+ * drops the links to it; linking and destroying must not race with steps on
+ * other threads. */
+SKIPCONV_API int skipconv_link_inputs(skipconv_handle h, skipconv_handle producer_x, skipconv_handle producer_sc);
+
 /* The same step on host buffers: copies x_t (host, [n][h][w][c_in] dtype;
  * pinned memory makes the copy asynchronous DMA) to the device, runs the
  * step, copies the whole z back to z_out (host float32 [n][ho][wo][c_out],

@@ -139,7 +139,7 @@ static void free_buffers(Layer* L)
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
                     L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag,
-                    L->pix_taps, L->gphi, L->w_loc};
+                    L->pix_taps, L->gphi, L->w_loc, L->ychg, L->tile_chg};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);
@@ -204,6 +204,18 @@ struct skipconv_s {
 };
 
 static Layer* get(skipconv_handle h) { return h ? &h->L : nullptr; }
+
+// Live layers, so that destroying a layer can drop the links other layers hold to it.
+static std::mutex& live_mu()
+{
+    static std::mutex mu;
+    return mu;
+}
+static std::vector<Layer*>& live_layers()
+{
+    static std::vector<Layer*> v;
+    return v;
+}
 
 extern "C" {
 
@@ -386,6 +398,10 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         delete h;
         return st;
     }
+    {
+        std::lock_guard<std::mutex> lock(live_mu());
+        live_layers().push_back(&h->L);
+    }
     *out = h;
     return SKIPCONV_OK;
 }
@@ -405,6 +421,7 @@ int skipconv_reset_state(skipconv_handle h)
     if (e == cudaSuccess && L->sched) e = cudaMemsetAsync(L->sched, 0, 16 * sizeof(int), L->stream);
     if (e == cudaSuccess) e = launch_reset_z(*L);
     if (e == cudaSuccess && L->y) e = cudaMemsetAsync(L->y, 0, (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * L->esize, L->stream);
+    if (e == cudaSuccess && L->tile_chg) e = cudaMemsetAsync(L->tile_chg, 0, 2 * (size_t)L->ntiles, L->stream);
     if (e != cudaSuccess) return status_of(e);
     L->t = 0;
     L->key = 1;
@@ -432,14 +449,25 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     const int force = (L->key || L->p.dense_mode) ? 1 : 0;
     if (L->fused) {
         const int kind = L->fused == 1 ? 4 : 5;
+        // stack propagation: a linked producer's change flags describe this x_t (or shortcut) only
+        // when it is that producer's y and the producer stepped exactly once since this layer did
+        const Layer* px = (L->link_x && x_t == L->link_x->y && L->link_x->steps == L->link_x_seen + 1) ? L->link_x
+                                                                                                      : nullptr;
+        const Layer* psc = (shortcut && L->link_sc && shortcut == L->link_sc->y &&
+                            L->link_sc->steps == L->link_sc_seen + 1)
+                               ? L->link_sc
+                               : nullptr;
         const int slot = prof_begin(L, kind);
         const cudaError_t e = L->fused == 1 ? launch_step_fused(*L, x_t, force)
-                                            : launch_step_local(*L, x_t, shortcut, force);
+                                            : launch_step_local(*L, x_t, shortcut, force, px, psc);
         prof_end(L, slot);
         if (e != cudaSuccess) return status_of(e);
         L->since_key = force && L->key ? 1 : L->since_key + 1;
         L->t += 1;
         L->key = 0;
+        L->steps += 1;
+        if (L->link_x) L->link_x_seen = L->link_x->steps;
+        if (L->link_sc) L->link_sc_seen = L->link_sc->steps;
         return SKIPCONV_OK;
     }
     const bool gumbel = L->p.gate == SKIPCONV_GATE_GUMBEL;
@@ -468,6 +496,46 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     L->since_key = force && L->key ? 1 : L->since_key + 1;
     L->t += 1;
     L->key = 0;
+    L->steps += 1;
+    return SKIPCONV_OK;
+}
+
+int skipconv_link_inputs(skipconv_handle h, skipconv_handle producer_x, skipconv_handle producer_sc)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    Layer* px = get(producer_x);
+    Layer* psc = get(producer_sc);
+    if (px == L || psc == L) return set_error("a layer cannot be linked to itself"), SKIPCONV_ERR_INVALID;
+    if (!px && psc) return set_error("a shortcut link needs the x_t link"), SKIPCONV_ERR_INVALID;
+    if (px) {
+        if (L->fused != 2 || !L->local_staged)
+            return set_error("stack propagation needs this layer on the one-launch CUDA-core step"),
+                   SKIPCONV_ERR_UNSUPPORTED;
+        for (const Layer* P : {px, psc}) {
+            if (!P) continue;
+            if (P->fused != 2 || !P->ychg)
+                return set_error("a linked producer must keep y and run the one-launch CUDA-core step"),
+                       SKIPCONV_ERR_UNSUPPORTED;
+            if (P->stream != L->stream) return set_error("linked layers must share the stream"), SKIPCONV_ERR_INVALID;
+            if (P->p.n_streams != L->p.n_streams || P->p.dtype != L->p.dtype)
+                return set_error("linked layers differ in streams or dtype"), SKIPCONV_ERR_INVALID;
+        }
+        if (px->ho != L->p.h || px->wo != L->p.w || px->p.c_out != L->p.c_in)
+            return set_error("x_t producer's y is [n][%d][%d][%d], this layer's x_t [n][%d][%d][%d]", px->ho, px->wo,
+                             px->p.c_out, L->p.h, L->p.w, L->p.c_in),
+                   SKIPCONV_ERR_INVALID;
+        if (psc && (psc->ho != L->ho || psc->wo != L->wo || psc->p.c_out != L->p.c_out))
+            return set_error("shortcut producer's y is [n][%d][%d][%d], this layer's output [n][%d][%d][%d]", psc->ho,
+                             psc->wo, psc->p.c_out, L->ho, L->wo, L->p.c_out),
+                   SKIPCONV_ERR_INVALID;
+    }
+    std::lock_guard<std::mutex> lock(live_mu());
+    L->link_x = px;
+    L->link_sc = psc;
+    // the first step that may use a link is the one after the producer's next step
+    L->link_x_seen = px ? px->steps : 0;
+    L->link_sc_seen = psc ? psc->steps : 0;
     return SKIPCONV_OK;
 }
 
@@ -526,6 +594,19 @@ int skipconv_destroy(skipconv_handle h)
 {
     if (!h) return SKIPCONV_OK;
     Layer* L = get(h);
+    {
+        std::lock_guard<std::mutex> lock(live_mu());
+        auto& v = live_layers();
+        for (size_t i = 0; i < v.size();) {
+            if (v[i] == L) {
+                v[i] = v.back();
+                v.pop_back();
+                continue;
+            }
+            if (v[i]->link_x == L || v[i]->link_sc == L) v[i]->link_x = v[i]->link_sc = nullptr;
+            ++i;
+        }
+    }
     cudaError_t e = cudaStreamSynchronize(L->stream);
     int st = e == cudaSuccess ? check_device_word(L) : status_of(e);
     free_buffers(L);

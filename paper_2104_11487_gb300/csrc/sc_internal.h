@@ -83,6 +83,16 @@ struct Layer {
     CUtensorMap tmap_fp[2]; // footprint boxes of the two state frames
     CUtensorMap tmap_ztile; // tile boxes of z
     void* w_loc;            // weights packed per CTA slice, layer dtype
+    uint8_t* ychg;          // per gate block: the last step may have changed y (layers with y)
+    uint8_t* tile_chg;      // [2][tiles]: some owned input pixel's change flag is set in chg[parity]
+    int ntiles;             // tiles of the staged form
+
+    // stack propagation (skipconv_link_inputs): the layers whose y this layer takes as x_t and as
+    // the shortcut, and their step counts when this layer last stepped
+    struct Layer* link_x;
+    struct Layer* link_sc;
+    long long link_x_seen, link_sc_seen;
+    long long steps;        // steps since create (never reset)
 };
 
 // ------------------------------------------------------------------ launchers
@@ -135,7 +145,10 @@ constexpr double LOCAL_AUTO_MAX_MACS = 67108864.0;   // 2^26
 bool step_local_preferred(const Layer& L);
 bool step_local_supported(const Layer& L);
 cudaError_t step_local_prepare(Layer& L);
-cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* shortcut, int force);
+// px / psc: the linked producers of x_t / of the shortcut whose y-change flags
+// are valid for this step (NULL: not linked, or not valid for this step).
+cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, int force, const Layer* px,
+                              const Layer* psc);
 
 // Driver entry point for tensor-map encoding (resolved once through the runtime).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

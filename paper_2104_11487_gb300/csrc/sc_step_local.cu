@@ -67,6 +67,9 @@ struct LocalArgs {
     int n, H, W, C, Ho, Wo, Co, KH, KW, stride, pad, b, nby, nbx, cpg, opg, groups, act;
     int sb, nty, ntx, FH, FW, CP;
     float thr;                 // threshold on the raw local l1 sum
+    uint8_t* ychg;             // per block: this step may change y (NULL without y)
+    const uint8_t* psc_chg;    // the shortcut's producer's flags (NULL: unknown, assume changed)
+    int pscb, pscnby, pscnbx;
 };
 
 __device__ __forceinline__ unsigned bits_of(float v) { return __float_as_uint(v); }
@@ -84,6 +87,21 @@ __device__ __forceinline__ float warp_max(float v)
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
     return v;
+}
+
+// Whether any of a producer's gate blocks over rows [r0, r1) x columns [c0, c1)
+// of stream nn flagged a change (every thread of the CTA calls it; returns the
+// calling thread's share, to be combined with __syncthreads_or).
+__device__ __forceinline__ int any_block_flag(const uint8_t* flags, int b, int nby, int nbx, int nn, int r0, int r1,
+                                              int c0, int c1, int tid, int nthreads)
+{
+    if (r1 <= r0 || c1 <= c0) return 0;
+    const int by0 = r0 / b, bx0 = c0 / b;
+    const int nbw = (c1 - 1) / b - bx0 + 1, nbb = ((r1 - 1) / b - by0 + 1) * nbw;
+    int any = 0;
+    for (int q = tid; q < nbb; q += nthreads)
+        any |= flags[((size_t)nn * nby + by0 + q / nbw) * nbx + bx0 + q % nbw];
+    return any;
 }
 
 template <typename T, bool DW, bool V4>
@@ -191,7 +209,18 @@ __global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
             }
             best = warp_max(best);
             open = (a.force || best > a.thr) ? 1 : 0;
-            if (lane == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
+            if (lane == 0) {
+                a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
+                if (a.ychg) {
+                    int yc = open;
+                    if (!yc && a.sc)
+                        yc = a.psc_chg == nullptr ? 1
+                                                  : any_block_flag(a.psc_chg, a.pscb, a.pscnby, a.pscnbx, nn, by * a.b,
+                                                                   min(a.Ho, (by + 1) * a.b), bx * a.b,
+                                                                   min(a.Wo, (bx + 1) * a.b), 0, 1);
+                    a.ychg[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)(yc != 0);
+                }
+            }
         }
         if (lane == 0) s_open[bq] = open;
     }
@@ -345,7 +374,17 @@ struct FastArgs {
     int sb, nty, ntx, FH, FW, CP, nsl, K;
     uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq;   // byte offsets
     float thr;
+    // stack propagation
+    const uint8_t* px_chg;       // the layer that produced x_t: its per-block "y may have changed" flags
+    int pxb, pxnby, pxnbx;       //   (NULL when x_t is not a linked layer's y of the step just before)
+    const uint8_t* psc_chg;      // the same for the shortcut's producer
+    int pscb, pscnby, pscnbx;
+    uint8_t* ychg;               // this layer's per-block y-change flags (NULL without y)
+    const uint8_t* tile_chg_prev;  // per tile: some owned pixel changed at the previous step
+    uint8_t* tile_chg_cur;       // per tile: some owned pixel changes at this step
 };
+
+
 
 __device__ __forceinline__ float4 load_w4(const float* w) { return *reinterpret_cast<const float4*>(w); }
 __device__ __forceinline__ float4 load_w4(const __nv_bfloat16* w)
@@ -398,6 +437,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
     __shared__ int s_open[MAX_TILE_BLOCKS];
     __shared__ int s_max[MAX_TILE_BLOCKS];      // per gate block: largest support sum (float bits)
     __shared__ int s_nloc;
+    __shared__ int s_tchg;                      // some owned pixel changed at this step
     uint8_t* base = align_smem_1024(smem_raw);
     const T* Xt = reinterpret_cast<const T*>(base);
     const T* Xp = reinterpret_cast<const T*>(base + a.off_xp);
@@ -437,9 +477,51 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         prefetch_tmap(&tm_xt);
         prefetch_tmap(&tm_xp);
         s_nloc = 0;
+        s_tchg = 0;
     }
     if (tid < MAX_TILE_BLOCKS) s_max[tid] = 0;
     grid_dependency_wait();
+    if (blockIdx.x == 0 && tid == 0) *a.count_next = 0;
+    // owned input pixels of this tile (every input pixel has exactly one owner tile)
+    const int own_y0 = min(ty * span * a.stride, a.H);
+    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
+    const int own_x0 = min(tx * span * a.stride, a.W);
+    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
+    const int oww = own_x1 - own_x0, npx = (own_y1 - own_y0) * oww;
+    if (a.px_chg != nullptr && !a.force) {
+        // stack propagation: x_t is a linked layer's y, which changed only in the blocks that layer
+        // flagged.  If none under this tile's footprint and owned pixels changed, no owned pixel
+        // changed at the previous step either, and the shortcut did not change over the tile, then
+        // r_t = 0 over the footprint: every block stays closed and there is nothing to commit or
+        // refresh -- the full step's outcome, without reading the tile.
+        int any = (tid == 0 && a.tile_chg_prev[tile]) ? 1 : 0;
+        any |= any_block_flag(a.px_chg, a.pxb, a.pxnby, a.pxnbx, nn, max(0, min(fy0, own_y0)),
+                              min(a.H, max(fy0 + a.FH, own_y1)), max(0, min(fx0, own_x0)),
+                              min(a.W, max(fx0 + a.FW, own_x1)), tid, FT);
+        if (has_sc) {
+            if (a.psc_chg == nullptr) any = 1;
+            else any |= any_block_flag(a.psc_chg, a.pscb, a.pscnby, a.pscnbx, nn, oy0, min(a.Ho, oy0 + span), ox0,
+                                       min(a.Wo, ox0 + span), tid, FT);
+        }
+        if (!__syncthreads_or(any)) {
+            if (sl == 0) {
+                for (int bq = tid; bq < a.sb * a.sb; bq += FT) {
+                    const int by = ty * a.sb + bq / a.sb, bx = tx * a.sb + bq % a.sb;
+                    if (by < a.nby && bx < a.nbx) {
+                        a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = 0;
+                        if (a.ychg) a.ychg[((size_t)nn * a.nby + by) * a.nbx + bx] = 0;
+                    }
+                }
+                if (a.tile_chg_cur[tile]) {   // this parity's flags still hold two steps ago's changes
+                    for (int q = tid; q < npx; q += FT)
+                        a.chg_cur[((size_t)nn * a.H + own_y0 + q / oww) * a.W + own_x0 + q % oww] = 0;
+                    if (tid == 0) a.tile_chg_cur[tile] = 0;
+                }
+            }
+            if (tid == 0) mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);   // the weight copy in flight
+            return;
+        }
+    }
     if (tid == 0) {
         mbar_arrive_expect_tx(bar_x, 2u * (uint32_t)FP * (uint32_t)a.C * (uint32_t)sizeof(T));
         tma_load_4d(smem_u32(Xt), &tm_xt, bar_x, 0, fx0, fy0, nn);
@@ -452,15 +534,8 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         }
     }
     grid_launch_dependents();
-    if (blockIdx.x == 0 && tid == 0) *a.count_next = 0;
 
-    // owned input pixels of this tile (every input pixel has exactly one owner tile) and, for
-    // slice 0, their change flags of the previous step
-    const int own_y0 = min(ty * span * a.stride, a.H);
-    const int own_y1 = ty == a.nty - 1 ? a.H : min((ty + 1) * span * a.stride, a.H);
-    const int own_x0 = min(tx * span * a.stride, a.W);
-    const int own_x1 = tx == a.ntx - 1 ? a.W : min((tx + 1) * span * a.stride, a.W);
-    const int oww = own_x1 - own_x0, npx = (own_y1 - own_y0) * oww;
+    // slice 0: the owned pixels' change flags of the previous step
     if (sl == 0)
         for (int q = tid; q < npx; q += FT)
             chgs[q] = a.chg_prev[((size_t)nn * a.H + own_y0 + q / oww) * a.W + own_x0 + q % oww];
@@ -529,7 +604,10 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             const bool changed = Dq[fq] != 0;
             if (changed || chgs[q])
                 (reinterpret_cast<uint4*>(xn) + pix * CH)[k] = reinterpret_cast<const uint4*>(Xt + (size_t)fq * a.C)[k];
-            if (k == 0) a.chg_cur[pix] = changed ? 1 : 0;
+            if (k == 0) {
+                a.chg_cur[pix] = changed ? 1 : 0;
+                if (changed) s_tchg = 1;
+            }
         }
         const T* xt = static_cast<const T*>(a.xt);
         const T* xp = static_cast<const T*>(a.xp);
@@ -542,7 +620,10 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             const bool changed = __any_sync(0xffffffffu, d != 0);
             if (changed || chgs[q])
                 for (int c = lane; c < a.C; c += 32) xn[pix * a.C + c] = xt[pix * a.C + c];
-            if (lane == 0) a.chg_cur[pix] = changed ? 1 : 0;
+            if (lane == 0) {
+                a.chg_cur[pix] = changed ? 1 : 0;
+                if (changed) s_tchg = 1;
+            }
         }
     }
 
@@ -574,8 +655,19 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             if (sl == 0) a.mask[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)open;
         }
         s_open[tid] = open;
+        // this layer's y may change where a block is open, or (with a shortcut) where the shortcut did
+        if (sl == 0 && a.ychg && by < a.nby && bx < a.nbx) {
+            int yc = open;
+            if (!yc && has_sc)
+                yc = a.psc_chg == nullptr
+                         ? 1
+                         : any_block_flag(a.psc_chg, a.pscb, a.pscnby, a.pscnbx, nn, by * a.b, min(a.Ho, (by + 1) * a.b),
+                                          bx * a.b, min(a.Wo, (bx + 1) * a.b), 0, 1);
+            a.ychg[((size_t)nn * a.nby + by) * a.nbx + bx] = (uint8_t)(yc != 0);
+        }
     }
     __syncthreads();
+    if (sl == 0 && tid == 0) a.tile_chg_cur[tile] = (uint8_t)s_tchg;
     bool any_open = false;
     for (int bq = 0; bq < a.sb * a.sb; ++bq) any_open |= s_open[bq] != 0;
     if (tid == 0 && any_open && !has_sc) {
@@ -984,6 +1076,21 @@ bool step_local_supported(const Layer& L)
     return staged_ok(L, nullptr) || choose_shape(L).smem <= LOCAL_MAX_SMEM;
 }
 
+// Layers that keep y publish, per gate block, whether a step may have changed it
+// (read by linked consumers).  All ones until the first step (a key frame).
+static cudaError_t alloc_ychg(Layer& L)
+{
+    if (!L.y) return cudaSuccess;
+    const size_t nblk = (size_t)L.p.n_streams * L.nby * L.nbx;
+    cudaError_t e = cudaMalloc((void**)&L.ychg, nblk);
+    if (e != cudaSuccess) {
+        L.ychg = nullptr;
+        return e;
+    }
+    L.state_bytes += nblk;
+    return cudaMemsetAsync(L.ychg, 1, nblk, L.stream);
+}
+
 cudaError_t step_local_prepare(Layer& L)
 {
     StagedShape t;
@@ -1016,13 +1123,26 @@ cudaError_t step_local_prepare(Layer& L)
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         L.local_staged = 1;
+        L.ntiles = (int)((long long)L.p.n_streams * ((L.nby + t.g.sb - 1) / t.g.sb) * ((L.nbx + t.g.sb - 1) / t.g.sb));
+        e = cudaMalloc((void**)&L.tile_chg, 2 * (size_t)L.ntiles);
+        if (e != cudaSuccess) {
+            L.tile_chg = nullptr;
+            return e;
+        }
+        L.state_bytes += 2 * (size_t)L.ntiles;
+        e = cudaMemsetAsync(L.tile_chg, 0, 2 * (size_t)L.ntiles, L.stream);
+        if (e == cudaSuccess) e = alloc_ychg(L);
+        if (e != cudaSuccess) return e;
         return ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
     }
     L.local_staged = 0;
+    const cudaError_t e = alloc_ychg(L);
+    if (e != cudaSuccess) return e;
     return ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
 }
 
-cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* shortcut, int force)
+cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, int force, const Layer* px,
+                              const Layer* psc)
 {
     const int cur = (int)(L.t & 1), nxt = cur ^ 1;
     cudaLaunchAttribute attr[1];
@@ -1061,6 +1181,13 @@ cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* short
         a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
         a.off_scr = t.off_scr; a.off_z = t.off_z; a.off_sc = t.off_sc; a.off_chg = t.off_chg; a.off_dq = t.off_dq;
         a.thr = L.gate_thr;
+        a.px_chg = px ? px->ychg : nullptr;
+        a.pxb = px ? px->p.block : 1; a.pxnby = px ? px->nby : 1; a.pxnbx = px ? px->nbx : 1;
+        a.psc_chg = psc ? psc->ychg : nullptr;
+        a.pscb = psc ? psc->p.block : 1; a.pscnby = psc ? psc->nby : 1; a.pscnbx = psc ? psc->nbx : 1;
+        a.ychg = L.ychg;
+        a.tile_chg_prev = L.tile_chg + (size_t)nxt * L.ntiles;
+        a.tile_chg_cur = L.tile_chg + (size_t)cur * L.ntiles;
         alignas(64) CUtensorMap tm_sc = L.tmap_ztile;   // unused without a shortcut
         if (a.sc && !encode_tile_map(&tm_sc, a.sc, L, t, false)) {
             set_error("tensor map of the shortcut rejected");
@@ -1097,6 +1224,10 @@ cudaError_t launch_step_local(const Layer& L, const void* x_t, const void* short
     a.ntx = (L.nbx + s.sb - 1) / s.sb;
     a.FH = s.FH; a.FW = s.FW; a.CP = s.CP;
     a.thr = L.gate_thr;
+    a.ychg = L.ychg;
+    a.psc_chg = psc ? psc->ychg : nullptr;
+    a.pscb = psc ? psc->p.block : 1; a.pscnby = psc ? psc->nby : 1; a.pscnbx = psc ? psc->nbx : 1;
+    (void)px;   // the general form reads every tile (it does not skip)
     const long long tiles = (long long)a.n * a.nty * a.ntx;
     if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = pdl_config(L, tiles, LT, s.smem, attr);

@@ -84,6 +84,12 @@ def skipconv_set_gate_weights(handle: int, phi_oihw, phi_bias: float = 0.0) -> N
     check("skipconv_set_gate_weights", _lib.lib().skipconv_set_gate_weights(handle, _ptr(phi_oihw), float(phi_bias)))
 
 
+def skipconv_link_inputs(handle: int, producer_x: int | None, producer_sc: int | None = None) -> None:
+    """Stack propagation: this layer's x_t is producer_x's y (and its shortcut
+    producer_sc's y); see include/skipconv.h.  producer_x = None unlinks."""
+    check("skipconv_link_inputs", _lib.lib().skipconv_link_inputs(handle, producer_x, producer_sc))
+
+
 def skipconv_get_info(handle: int) -> Info:
     info = Info()
     check("skipconv_get_info", _lib.lib().skipconv_get_info(handle, ctypes.byref(info)))
@@ -171,6 +177,12 @@ class SkipConvLayer:
 
     def reset(self) -> None:
         skipconv_reset_state(self.handle)
+
+    def link(self, producer_x=None, producer_sc=None) -> None:
+        """Stack propagation: x_t will be producer_x.y() (and the shortcut
+        producer_sc.y()) at every step; None unlinks."""
+        skipconv_link_inputs(self.handle, None if producer_x is None else producer_x.handle,
+                             None if producer_sc is None else producer_sc.handle)
 
     def z(self):
         return self._view(skipconv_get_z(self.handle), self.shape_out, self.torch.float32)

@@ -142,7 +142,20 @@ def c4(density: float = 0.10, T: int = 32, n: int = 8, h: int = 128, w: int = 12
     return Workload("c4", dtype, n, h, w, c, T, layers, ws, bs, frames)
 
 
-WORKLOADS = {"c0": c0, "c1": c1, "c2": c2, "c3": c3, "c4": c4}
+def dw3(density: float = 0.10, T: int = 16, n: int = 8, h: int = 128, w: int = 128, c: int = 128,
+        block: int = 8) -> Workload:
+    """A frame-sized stack for stack propagation: three depthwise 3x3 layers
+    (c channels, ReLU between) on c4's block-perturbation video -- each layer
+    streams two 32 MiB frames per step in full, while only the perturbed blocks
+    and their halo change.  `frames` is an iterable yielding (t, frame)."""
+    layers = [LayerDef(c, c, 3, 1, 1, c, block, 0.05, ACT_RELU, name="dw%d" % i) for i in range(3)]
+    n_changed = int(round(density * (h // block) * (w // block)))
+    frames = block_perturbation_video(5000, T, n, h, w, c, block, n_changed, bf16=True)
+    ws, bs = _weights(5001, layers, bf16=True, bias_std=0.01)
+    return Workload("dw3", "bf16", n, h, w, c, T, layers, ws, bs, frames)
+
+
+WORKLOADS = {"c0": c0, "c1": c1, "c2": c2, "c3": c3, "c4": c4, "dw3": dw3}
 
 
 def make_workload(name: str, **kw) -> Workload:
