@@ -89,6 +89,9 @@ def lib():
         L.oc_step_sampled.argtypes = [PP, _DP, _DP, ctypes.c_double, _DP, _DP, ctypes.c_int, _IP, _DP, ctypes.c_int,
                                       _UP]
         L.oc_step_sampled.restype = ctypes.c_long
+        L.oc_warp.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _DP, _DP, _DP]
+        L.oc_step_warped.argtypes = [PP, _DP, _DP, ctypes.c_double, _DP, _DP, _DP, _DP, ctypes.c_int, _DP, _UP]
+        L.oc_step_warped.restype = ctypes.c_long
         L.oc_round_bf16.argtypes = [ctypes.c_double]
         L.oc_round_bf16.restype = ctypes.c_double
         L.oc_layer_output.argtypes = [ctypes.c_size_t, _DP, _DP, ctypes.c_int, ctypes.c_int, _DP]
@@ -238,6 +241,39 @@ class OracleLayer:
             raise MemoryError("oracle step: allocation failed")
         self.key = False
         return score, mask
+
+    def step_warped(self, x_t, flow, force: bool | None = None):
+        """Advance one frame with a warped residual (Sec. 3.4, Eq. 10-11):
+        r_t = x_t - T(x_{t-1}), z~_t = T~(z~_{t-1}) + g (.) (w * r_t), T and T~
+        bilinear with the per-pixel flow [n, h, w, 2] = (dy, dx).  A key frame
+        has no previous frame to warp: it is the plain key-frame step."""
+        if self.key:
+            return self.step(x_t, force)
+        s = self.spec
+        x_t = _f64(x_t)
+        flow = _f64(flow)
+        assert x_t.shape == self.x_prev.shape and flow.shape == (s.n, s.h, s.w, 2)
+        score = np.empty((s.n, s.ho, s.wo), np.float64)
+        mask = np.empty((s.n, s.nby, s.nbx), np.uint8)
+        f = self.dense_mode if force is None else force
+        rc = lib().oc_step_warped(ctypes.byref(s.params()), _dp(self.w), _dp(self.phi), self.phi_bias, _dp(x_t),
+                                  _dp(self.x_prev), _dp(self.z), _dp(flow), int(f), _dp(score),
+                                  mask.ctypes.data_as(_UP))
+        if rc == -2:
+            raise ValueError("warped residuals need a layer that keeps the frame size (stride 1, same padding)")
+        if rc < 0:
+            raise MemoryError("oracle step: allocation failed")
+        return score, mask
+
+
+def warp(x, flow):
+    """T of Sec. 3.4: x [n, h, w, c] sampled at p + flow(p) by bilinear interpolation, zero outside."""
+    x = _f64(x)
+    flow = _f64(flow)
+    n, h, w, c = x.shape
+    out = np.empty_like(x)
+    lib().oc_warp(n, h, w, c, _dp(flow), _dp(x), _dp(out))
+    return out
 
 
 class SampledOracleLayer:

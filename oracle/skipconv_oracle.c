@@ -276,6 +276,93 @@ long oc_step(const oc_params* p, const double* w, const double* phi, double phi_
     return open;
 }
 
+/* Warp T of Sec. 3.4 (Eq. 10-11): out(n, y, x, c) = in sampled at
+ * (y + dy, x + dx), (dy, dx) = flow[n][y][x], by bilinear interpolation of the
+ * four surrounding pixels; a pixel outside the frame contributes zero.  in and
+ * out are [n][H][W][C]; flow is [n][H][W][2] (dy, dx) in pixels. */
+void oc_warp(int n, int H, int W, int C, const double* flow, const double* in, double* out)
+{
+#ifdef _OPENMP
+#pragma omp parallel for collapse(2) schedule(static)
+#endif
+    for (int ni = 0; ni < n; ++ni)
+        for (int y = 0; y < H; ++y)
+            for (int x = 0; x < W; ++x) {
+                const double* f = flow + (((size_t)ni * H + y) * W + x) * 2;
+                const double sy = y + f[0], sx = x + f[1];
+                const double fy = floor(sy), fx = floor(sx);
+                const double ay = sy - fy, ax = sx - fx;
+                const int y0 = (int)fy, x0 = (int)fx;
+                const int ys[4] = {y0, y0, y0 + 1, y0 + 1}, xs[4] = {x0, x0 + 1, x0, x0 + 1};
+                const double wt[4] = {(1.0 - ay) * (1.0 - ax), (1.0 - ay) * ax, ay * (1.0 - ax), ay * ax};
+                for (int c = 0; c < C; ++c) {
+                    double v = 0.0;
+                    for (int q = 0; q < 4; ++q)
+                        if (ys[q] >= 0 && ys[q] < H && xs[q] >= 0 && xs[q] < W)
+                            v += wt[q] * in[(((size_t)ni * H + ys[q]) * W + xs[q]) * C + c];
+                    out[(((size_t)ni * H + y) * W + x) * C + c] = v;
+                }
+            }
+}
+
+/* Skip-Conv step with a warped residual (Sec. 3.4, Eq. 10-11): the residual
+ * is taken against the previous input warped by T,
+ *     r_t = x_t - T(x_{t-1}),
+ * and the output is decoded by warping the previous output with the same
+ * flow before adding the gated convolution of the residual,
+ *     z~_t = T~(z~_{t-1}) + g(r_t) (.) (w * r_t),
+ * then x_{t-1} <- x_t.  T~ applies the flow on the output grid, so the layer
+ * must keep the frame size (stride 1, ho = h, wo = w).  The gate, blocks and
+ * force are those of oc_step.  Returns the number of open blocks, -1 on
+ * allocation failure, -2 when the output grid differs from the input grid. */
+long oc_step_warped(const oc_params* p, const double* w, const double* phi, double phi_bias, const double* x_t,
+                    double* x_prev, double* z, const double* flow, int force, double* score_out,
+                    unsigned char* mask_out)
+{
+    const int ho = oc_out_h(p), wo = oc_out_w(p);
+    if (p->stride != 1 || ho != p->h || wo != p->w) return -2;
+    const int nby = oc_blocks_y(p), nbx = oc_blocks_x(p), b = p->block;
+    size_t nx = (size_t)p->n * p->h * p->w * p->c_in;
+    size_t nz = (size_t)p->n * ho * wo * p->c_out;
+    double* tx = (double*)malloc(nx * sizeof(double));
+    double* r = (double*)malloc(nx * sizeof(double));
+    double* zw = (double*)malloc(nz * sizeof(double));
+    double* score = score_out ? score_out : (double*)malloc((size_t)p->n * ho * wo * sizeof(double));
+    unsigned char* mask = mask_out ? mask_out : (unsigned char*)malloc((size_t)p->n * nby * nbx);
+    if (!tx || !r || !zw || !score || !mask) {
+        free(tx);
+        free(r);
+        free(zw);
+        if (!score_out) free(score);
+        if (!mask_out) free(mask);
+        return -1;
+    }
+    oc_warp(p->n, p->h, p->w, p->c_in, flow, x_prev, tx);    /* T(x_{t-1}) */
+    oc_residual(p, x_t, tx, r);                              /* r_t = x_t - T(x_{t-1}) */
+    gate_scores_of(p, w, r, phi, phi_bias, score);
+    oc_block_gate(p, score, force, mask);
+    oc_warp(p->n, ho, wo, p->c_out, flow, z, zw);            /* T~(z~_{t-1}) */
+    memcpy(z, zw, nz * sizeof(double));
+#ifdef _OPENMP
+#pragma omp parallel for collapse(2) schedule(dynamic)
+#endif
+    for (int n = 0; n < p->n; ++n)
+        for (int i = 0; i < ho; ++i)
+            for (int j = 0; j < wo; ++j) {
+                if (!mask[((size_t)n * nby + i / b) * nbx + j / b]) continue;
+                for (int o = 0; o < p->c_out; ++o) z[ix_z(p, n, i, j, o)] += conv_at(p, w, r, n, i, j, o);
+            }
+    memcpy(x_prev, x_t, nx * sizeof(double));
+    long open = 0;
+    for (size_t k = 0; k < (size_t)p->n * nby * nbx; ++k) open += mask[k];
+    free(tx);
+    free(r);
+    free(zw);
+    if (!score_out) free(score);
+    if (!mask_out) free(mask);
+    return open;
+}
+
 /* The same step, with z kept only at n_samples chosen output locations
  * (z_samples is [n_samples][c_out], locations given as (n, i, j) triples).
  * The gate is evaluated over the whole frame exactly as in oc_step, so the

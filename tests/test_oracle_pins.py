@@ -422,3 +422,124 @@ def test_gumbel_step_is_masked_dense_update(stride, block):
         closed += int((mask == 0).sum())
         np.testing.assert_allclose(lay.z, z, rtol=1e-12, atol=1e-12)
     assert closed > 0, "the case must close some gates"
+
+
+# ------------------------------------------------------- warped residuals (Eq. 10-11)
+def test_warp_is_library_grid_sample():
+    """T (bilinear, zero outside) equals torch's grid_sample with align_corners=True
+    and zero padding, sampled at p + flow(p)."""
+    rng = np.random.default_rng(71)
+    n, h, w, c = 2, 7, 9, 3
+    x = rng.standard_normal((n, h, w, c))
+    flow = rng.uniform(-2.5, 2.5, (n, h, w, 2))
+    got = oracle.warp(x, flow)
+    yy, xx = np.meshgrid(np.arange(h), np.arange(w), indexing="ij")
+    sy, sx = yy[None] + flow[..., 0], xx[None] + flow[..., 1]
+    grid = np.stack([2 * sx / (w - 1) - 1, 2 * sy / (h - 1) - 1], axis=-1)      # (x, y) in [-1, 1]
+    ref = F.grid_sample(torch.from_numpy(x).permute(0, 3, 1, 2), torch.from_numpy(grid), mode="bilinear",
+                        padding_mode="zeros", align_corners=True).permute(0, 2, 3, 1).numpy()
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+
+
+def test_warped_step_with_zero_flow_is_the_plain_step():
+    """f(x) = x - x_{t-1} is the special case T = identity (Sec. 3.4): with a zero
+    flow the warped step is the plain step, bit for bit."""
+    rng = np.random.default_rng(72)
+    spec = LayerSpec(n=2, c_in=3, c_out=4, h=9, w=8, k=3, block=2, eps=0.3)
+    w, b = rand_layer(rng, spec)
+    a, bb = OracleLayer(spec, w, b), OracleLayer(spec, w, b)
+    zero = np.zeros((spec.n, spec.h, spec.w, 2))
+    for t in range(5):
+        x = rng.standard_normal((spec.n, spec.h, spec.w, spec.c_in)) * (0.2 if t else 1.0)
+        s1, m1 = a.step(x)
+        s2, m2 = bb.step_warped(x, zero)
+        np.testing.assert_array_equal(m1, m2)
+        np.testing.assert_array_equal(s1, s2)
+        np.testing.assert_array_equal(a.z, bb.z)
+
+
+@pytest.mark.parametrize("d", [(1, -2), (0, 3), (-1, 1)])
+def test_warped_step_decodes_translations_exactly(d):
+    """Eq. 11 with an equivariant warp: for an integer translation and every gate
+    open, T~(z_{t-1}) + w * (x_t - T(x_{t-1})) = w * x_t + b at every location far
+    enough from the border (the warp's zero fill and the convolution's padding
+    differ near it), so the warped recurrence reproduces the dense output."""
+    rng = np.random.default_rng(73)
+    spec = LayerSpec(n=1, c_in=3, c_out=2, h=26, w=24, k=3, block=2, eps=0.0)
+    w, b = rand_layer(rng, spec)
+    lay = OracleLayer(spec, w, b)
+    flow = np.zeros((1, spec.h, spec.w, 2))
+    flow[..., 0], flow[..., 1] = d
+    T = 4
+    for t in range(T):
+        x = rng.standard_normal((1, spec.h, spec.w, spec.c_in))
+        _, m = lay.step_warped(x, flow)
+        assert m.all()
+    m = (T - 1) * max(abs(d[0]), abs(d[1])) + spec.pad + 1     # border band the error can reach after T steps
+    ref = torch_conv(spec, w, x, b)
+    inner = (slice(None), slice(m, spec.h - m), slice(m, spec.w - m))
+    assert ref[inner].size > 0
+    np.testing.assert_allclose(lay.z[inner], ref[inner], rtol=0, atol=1e-10 * np.abs(ref).max())
+    # and the border does differ (the reading is not vacuous)
+    assert np.abs(lay.z - ref).max() > 1e-6
+
+
+def test_warped_step_brute_force_tiny():
+    """The warped step written out with plain Python loops (bilinear weights of the
+    four neighbours, zero outside; support sums; block max; masked update)."""
+    rng = np.random.default_rng(74)
+    spec = LayerSpec(n=1, c_in=2, c_out=2, h=6, w=5, k=3, block=2, eps=0.4)
+    w, b = rand_layer(rng, spec)
+    lay = OracleLayer(spec, w, b)
+    x0 = rng.standard_normal((1, spec.h, spec.w, spec.c_in))
+    lay.step(x0)
+    z = lay.z.copy()
+    xp = x0.copy()
+    opened = []
+    for t in range(3):
+        x = xp + rng.standard_normal(xp.shape) * (0.6 if t != 1 else 0.05)
+        flow = rng.uniform(-1.6, 1.6, (1, spec.h, spec.w, 2))
+
+        def bil(a, y, xx, c):
+            y0, x0_ = int(np.floor(y)), int(np.floor(xx))
+            ay, ax = y - y0, xx - x0_
+            v = 0.0
+            for (yy, xq, wt) in ((y0, x0_, (1 - ay) * (1 - ax)), (y0, x0_ + 1, (1 - ay) * ax),
+                                 (y0 + 1, x0_, ay * (1 - ax)), (y0 + 1, x0_ + 1, ay * ax)):
+                if 0 <= yy < a.shape[1] and 0 <= xq < a.shape[2]:
+                    v += wt * a[0, yy, xq, c]
+            return v
+        r = np.zeros_like(x)
+        zw = np.zeros_like(z)
+        for i in range(spec.h):
+            for j in range(spec.w):
+                fy, fx = flow[0, i, j]
+                for c in range(spec.c_in):
+                    r[0, i, j, c] = x[0, i, j, c] - bil(xp, i + fy, j + fx, c)
+                for o in range(spec.c_out):
+                    zw[0, i, j, o] = bil(z, i + fy, j + fx, o)
+        score = np.zeros((spec.h, spec.w))
+        delta = np.zeros_like(z)
+        for i in range(spec.h):
+            for j in range(spec.w):
+                s = 0.0
+                for kh in range(3):
+                    for kw in range(3):
+                        yy, xq = i + kh - 1, j + kw - 1
+                        if 0 <= yy < spec.h and 0 <= xq < spec.w:
+                            s += np.abs(r[0, yy, xq]).sum()
+                            for o in range(spec.c_out):
+                                delta[0, i, j, o] += (w[o, :, kh, kw] * r[0, yy, xq]).sum()
+                score[i, j] = s / (spec.c_in * 9)
+        mask = np.zeros((3, 3), bool)
+        for by in range(3):
+            for bx in range(3):
+                mask[by, bx] = score[2 * by:2 * by + 2, 2 * bx:2 * bx + 2].max() > spec.eps
+        z = zw + delta * np.repeat(np.repeat(mask, 2, 0), 2, 1)[None, :spec.h, :spec.w, None]
+        xp = x
+        s_o, m_o = lay.step_warped(x, flow)
+        np.testing.assert_array_equal(m_o[0], mask)
+        np.testing.assert_allclose(s_o[0], score, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(lay.z, z, rtol=1e-12, atol=1e-12)
+        opened.append(int(mask.sum()))
+    assert any(0 < k < 9 for k in opened), opened   # some frame mixes open and closed blocks
