@@ -140,6 +140,21 @@ SKIPCONV_API int skipconv_reset_state(skipconv_handle h);
  * x_t and shortcut must stay valid until the stream reaches this work. */
 SKIPCONV_API int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut);
 
+/* One step with a warped residual (Sec. 3.4, Eq. 10-11): the residual is
+ * taken against the previous input warped by the flow, r_t = x_t - T(x_{t-1}),
+ * and the previous output is warped the same way before the gated convolution
+ * of r_t is added: z~_t = T~(z~_{t-1}) + g(r_t) (.) (w * r_t).  T samples at
+ * (y + dy, x + dx) by bilinear interpolation of the four surrounding pixels,
+ * a pixel outside the frame contributing zero; T~ does the same on the output
+ * grid, so the layer must keep the frame size (stride 1, ho = h, wo = w).
+ * flow: device float32 [n][h][w][2], (dy, dx) in pixels, 4-byte aligned.  A
+ * key frame has no previous frame to warp and is the plain key-frame step.
+ * Every location of z (and y) moves; the gate, list and x_{t-1} <- x_t are as
+ * in skipconv_step.  The first warped step allocates a copy of z.  Errors as
+ * skipconv_step, and UNSUPPORTED unless the layer runs the one-launch
+ * CUDA-core step and keeps the frame size. */
+SKIPCONV_API int skipconv_step_warped(skipconv_handle h, const void* x_t, const void* shortcut, const float* flow);
+
 /* Stack propagation: the input of layer l+1 changes only where layer l's
  * output changed (the residual of Eq. 2 is zero elsewhere).  Declares that
  * this layer's x_t is producer_x's y and, if producer_sc is not NULL, that

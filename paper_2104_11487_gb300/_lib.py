@@ -41,6 +41,7 @@ SIGNATURES = {
     "skipconv_gate_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "skipconv_set_gate_weights": (c_int, [c_void_p, c_void_p, c_float]),
     "skipconv_link_inputs": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "skipconv_step_warped": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
     "skipconv_status_string": (ctypes.c_char_p, [c_int]),
     "skipconv_last_error": (ctypes.c_char_p, []),
 }

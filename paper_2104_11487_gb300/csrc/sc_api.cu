@@ -139,7 +139,7 @@ static void free_buffers(Layer* L)
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
                     L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag,
-                    L->pix_taps, L->gphi, L->w_loc, L->ychg, L->tile_chg};
+                    L->pix_taps, L->gphi, L->w_loc, L->ychg, L->tile_chg, L->z_prev};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);
@@ -497,6 +497,60 @@ int skipconv_step(skipconv_handle h, const void* x_t, const void* shortcut)
     L->t += 1;
     L->key = 0;
     L->steps += 1;
+    return SKIPCONV_OK;
+}
+
+int skipconv_step_warped(skipconv_handle h, const void* x_t, const void* shortcut, const float* flow)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!x_t || !flow) return set_error("x_t and flow must not be NULL"), SKIPCONV_ERR_INVALID;
+    if ((uintptr_t)x_t % 16 || (uintptr_t)shortcut % 16 || (uintptr_t)flow % 4)
+        return set_error("x_t and shortcut must be 16-byte aligned, flow 4-byte aligned"), SKIPCONV_ERR_INVALID;
+    if (shortcut && !L->y) return set_error("shortcut given but the layer keeps no y (emit_y = 0)"), SKIPCONV_ERR_INVALID;
+    if (!step_local_warp_supported(*L))
+        return set_error("warped residuals need a layer on the one-launch CUDA-core step that keeps the frame "
+                         "size (stride 1, ho = h, wo = w)"),
+               SKIPCONV_ERR_UNSUPPORTED;
+    if (int st = check_device_word(L)) return st;
+    if (L->p.key_interval > 0 && !L->key && L->since_key >= L->p.key_interval) {
+        const int st = skipconv_reset_state(h);   // periodic key frame (Table 4)
+        if (st != SKIPCONV_OK) return st;
+    }
+    // a key frame has no previous frame to warp: it is the plain key-frame step
+    if (L->key) return skipconv_step(h, x_t, shortcut);
+    const size_t nz = (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out;
+    cudaError_t e = cudaSuccess;
+    if (!L->z_prev) {
+        e = cudaMalloc((void**)&L->z_prev, nz * sizeof(float));
+        if (e != cudaSuccess) {
+            L->z_prev = nullptr;
+            return status_of(e);
+        }
+        L->state_bytes += nz * sizeof(float);
+    }
+    const int cur = (int)(L->t & 1);
+    // z~_t = T~(z~_{t-1}) everywhere, then + w * r_t at the open blocks with r_t = x_t - T(x_{t-1})
+    int slot = prof_begin(L, 3);
+    e = cudaMemcpyAsync(L->z_prev, L->z, nz * sizeof(float), cudaMemcpyDeviceToDevice, L->stream);
+    if (e == cudaSuccess) e = launch_warp_z(*L, L->z_prev, flow, L->y != nullptr && !shortcut);
+    prof_end(L, slot);
+    if (e == cudaSuccess) {
+        slot = prof_begin(L, 5);
+        e = launch_step_local(*L, x_t, shortcut, L->p.dense_mode ? 1 : 0, nullptr, nullptr, flow);
+        prof_end(L, slot);
+    }
+    // y moved everywhere, and this form keeps no per-tile commit flags: tell linked layers (and this
+    // layer's next linked step) to read whole frames
+    if (e == cudaSuccess && L->ychg)
+        e = cudaMemsetAsync(L->ychg, 1, (size_t)L->p.n_streams * L->nby * L->nbx, L->stream);
+    if (e == cudaSuccess && L->tile_chg) e = cudaMemsetAsync(L->tile_chg + (size_t)cur * L->ntiles, 1, L->ntiles, L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    L->since_key += 1;
+    L->t += 1;
+    L->steps += 1;
+    if (L->link_x) L->link_x_seen = L->link_x->steps;
+    if (L->link_sc) L->link_sc_seen = L->link_sc->steps;
     return SKIPCONV_OK;
 }
 

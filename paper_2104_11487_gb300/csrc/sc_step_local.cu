@@ -70,7 +70,45 @@ struct LocalArgs {
     uint8_t* ychg;             // per block: this step may change y (NULL without y)
     const uint8_t* psc_chg;    // the shortcut's producer's flags (NULL: unknown, assume changed)
     int pscb, pscnby, pscnbx;
+    const float* flow;         // warped residual (Eq. 10-11): [n][h][w][2] (dy, dx), or NULL
 };
+
+// The previous input as a warped residual sees it at pixel (iy, ix): T(x_{t-1})
+// samples x_{t-1} at (iy + dy, ix + dx) by bilinear interpolation of the four
+// surrounding pixels, a pixel outside the frame contributing zero (Eq. 10-11).
+// Corner element offsets of channel 0, and their weights (0 outside).
+struct Bilinear {
+    size_t off[4];
+    float wt[4];
+};
+
+__device__ __forceinline__ Bilinear bilinear_of(const float* flow, int nn, int H, int W, int C, int iy, int ix)
+{
+    const size_t pix = ((size_t)nn * H + iy) * W + ix;
+    const float sy = (float)iy + flow[2 * pix], sx = (float)ix + flow[2 * pix + 1];
+    const float y0f = floorf(sy), x0f = floorf(sx);
+    const float ay = sy - y0f, ax = sx - x0f;
+    const int y0 = (int)y0f, x0 = (int)x0f;
+    const int ys[4] = {y0, y0, y0 + 1, y0 + 1}, xs[4] = {x0, x0 + 1, x0, x0 + 1};
+    const float w[4] = {(1.f - ay) * (1.f - ax), (1.f - ay) * ax, ay * (1.f - ax), ay * ax};
+    Bilinear b;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const bool in = ys[q] >= 0 && ys[q] < H && xs[q] >= 0 && xs[q] < W;
+        b.off[q] = in ? (((size_t)nn * H + ys[q]) * W + xs[q]) * C : 0;
+        b.wt[q] = in ? w[q] : 0.f;
+    }
+    return b;
+}
+
+template <typename T>
+__device__ __forceinline__ float warped_at(const T* xp, const Bilinear& b, int c)
+{
+    float v = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v += b.wt[q] * to_f32(xp[b.off[q] + c]);
+    return v;
+}
 
 __device__ __forceinline__ unsigned bits_of(float v) { return __float_as_uint(v); }
 __device__ __forceinline__ unsigned bits_of(__nv_bfloat16 v) { return (unsigned)__bfloat16_as_ushort(v); }
@@ -144,10 +182,19 @@ __global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
             const bool in = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
             const size_t base = in ? (((size_t)nn * a.H + iy) * a.W + ix) * a.C : 0;
             float s = 0.f;
-            for (int c = 0; c < a.C; ++c) {
-                const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
-                R[(size_t)q * a.CP + c] = r;
-                s += fabsf(r);
+            if (a.flow && in) {
+                const Bilinear bl = bilinear_of(a.flow, nn, a.H, a.W, a.C, iy, ix);
+                for (int c = 0; c < a.C; ++c) {
+                    const float r = to_f32(xt[base + c]) - warped_at(xp, bl, c);
+                    R[(size_t)q * a.CP + c] = r;
+                    s += fabsf(r);
+                }
+            } else {
+                for (int c = 0; c < a.C; ++c) {
+                    const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
+                    R[(size_t)q * a.CP + c] = r;
+                    s += fabsf(r);
+                }
             }
             P[q] = s;
         }
@@ -169,10 +216,19 @@ __global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
             const bool in = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
             const size_t base = in ? (((size_t)nn * a.H + iy) * a.W + ix) * a.C : 0;
             float s = 0.f;
-            for (int c = lane; c < a.C; c += 32) {
-                const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
-                R[(size_t)q * a.CP + c] = r;
-                s += fabsf(r);
+            if (a.flow && in) {
+                const Bilinear bl = bilinear_of(a.flow, nn, a.H, a.W, a.C, iy, ix);
+                for (int c = lane; c < a.C; c += 32) {
+                    const float r = to_f32(xt[base + c]) - warped_at(xp, bl, c);
+                    R[(size_t)q * a.CP + c] = r;
+                    s += fabsf(r);
+                }
+            } else {
+                for (int c = lane; c < a.C; c += 32) {
+                    const float r = in ? to_f32(xt[base + c]) - to_f32(xp[base + c]) : 0.f;
+                    R[(size_t)q * a.CP + c] = r;
+                    s += fabsf(r);
+                }
             }
             s = warp_sum(s);
             if (lane == 0) P[q] = s;
@@ -1069,6 +1125,12 @@ bool step_local_preferred(const Layer& L)
     return dense_macs <= LOCAL_AUTO_MAX_MACS && staged_ok(L, nullptr);
 }
 
+bool step_local_warp_supported(const Layer& L)
+{
+    return L.fused == 2 && L.p.stride == 1 && L.ho == L.p.h && L.wo == L.p.w &&
+           choose_shape(L).smem <= LOCAL_MAX_SMEM;
+}
+
 bool step_local_supported(const Layer& L)
 {
     if (L.path != SKIPCONV_PATH_CUDA_CORE || L.p.conv_path == SKIPCONV_PATH_CUDA_CORE_SEPARATE) return false;
@@ -1132,8 +1194,10 @@ cudaError_t step_local_prepare(Layer& L)
         L.state_bytes += 2 * (size_t)L.ntiles;
         e = cudaMemsetAsync(L.tile_chg, 0, 2 * (size_t)L.ntiles, L.stream);
         if (e == cudaSuccess) e = alloc_ychg(L);
-        if (e != cudaSuccess) return e;
-        return ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
+        if (e == cudaSuccess) e = ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
+        // warped steps run the general form
+        if (e == cudaSuccess && choose_shape(L).smem <= LOCAL_MAX_SMEM) e = ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
+        return e;
     }
     L.local_staged = 0;
     const cudaError_t e = alloc_ychg(L);
@@ -1142,11 +1206,11 @@ cudaError_t step_local_prepare(Layer& L)
 }
 
 cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, int force, const Layer* px,
-                              const Layer* psc)
+                              const Layer* psc, const float* flow)
 {
     const int cur = (int)(L.t & 1), nxt = cur ^ 1;
     cudaLaunchAttribute attr[1];
-    if (L.local_staged) {
+    if (L.local_staged && !flow) {   // warped residuals take the general form (its loads sample the warp)
         StagedShape t;
         if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
         alignas(64) CUtensorMap tm_xt;
@@ -1227,6 +1291,7 @@ cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, i
     a.ychg = L.ychg;
     a.psc_chg = psc ? psc->ychg : nullptr;
     a.pscb = psc ? psc->p.block : 1; a.pscnby = psc ? psc->nby : 1; a.pscnbx = psc ? psc->nbx : 1;
+    a.flow = flow;
     (void)px;   // the general form reads every tile (it does not skip)
     const long long tiles = (long long)a.n * a.nty * a.ntx;
     if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;

@@ -84,6 +84,11 @@ def skipconv_set_gate_weights(handle: int, phi_oihw, phi_bias: float = 0.0) -> N
     check("skipconv_set_gate_weights", _lib.lib().skipconv_set_gate_weights(handle, _ptr(phi_oihw), float(phi_bias)))
 
 
+def skipconv_step_warped(handle: int, x_t, flow, shortcut=None) -> None:
+    """A step with a warped residual (Eq. 10-11); flow: float32 [n, h, w, 2] (dy, dx) on the device."""
+    check("skipconv_step_warped", _lib.lib().skipconv_step_warped(handle, _ptr(x_t), _ptr(shortcut), _ptr(flow)))
+
+
 def skipconv_link_inputs(handle: int, producer_x: int | None, producer_sc: int | None = None) -> None:
     """Stack propagation: this layer's x_t is producer_x's y (and its shortcut
     producer_sc's y); see include/skipconv.h.  producer_x = None unlinks."""
@@ -174,6 +179,13 @@ class SkipConvLayer:
         if shortcut is not None:
             assert tuple(shortcut.shape) == self.shape_out and shortcut.dtype == self.dtype
         skipconv_step(self.handle, x_t, shortcut)
+
+    def step_warped(self, x_t, flow, shortcut=None) -> None:
+        """One step with a warped residual (Eq. 10-11): flow float32 [n, h, w, 2] = (dy, dx)."""
+        assert tuple(x_t.shape) == self.shape_in and x_t.dtype == self.dtype and x_t.is_contiguous()
+        n, h, w = self.shape_in[:3]
+        assert tuple(flow.shape) == (n, h, w, 2) and flow.dtype == self.torch.float32 and flow.is_contiguous()
+        skipconv_step_warped(self.handle, x_t, flow, shortcut)
 
     def reset(self) -> None:
         skipconv_reset_state(self.handle)
