@@ -62,7 +62,8 @@ def parse():
                     help="stack propagation for the stacked workloads: also time linked stacks (both), "
                          "link them throughout (on), or not at all (off)")
     ap.add_argument("--workloads-only", default=None, metavar="NAMES",
-                    help="run only these of the single-layer and stacked workloads (comma-separated, e.g. c2,c3) "
+                    help="run only these of the single-layer and stacked workloads (comma-separated, e.g. c2,c3; "
+                         "\"warped\" for the warped-residual pan) "
                          "and print their report; for profiling them")
     ap.add_argument("--no-flush", action="store_true",
                     help="no L2 flush between timed steps: each step streams 134 MB of frames, more than the L2")
@@ -500,6 +501,51 @@ def workloads_report(torch, flush, tc_peak, hbm, warmup=3, names=("c0", "c1", "c
             "workloads": report}
 
 
+# ------------------------------------------------------ warped residuals
+def warped_report(torch, flush, steps=12, warmup=3):
+    """Warped residuals (Eq. 10-11) under a camera pan: a 128x128x64 bf16
+    texture window moving by (1, 1) px per frame, one 3x3 64->64 layer with
+    8x8 blocks and eps 0.05 on the one-launch CUDA-core step.  The plain
+    residual changes everywhere; warped by the pan's flow, the previous frame
+    matches the current one except in the strip entering at the border.
+    Per mode: median step time (CUDA events, L2 flushed between steps) and the
+    mean open-block density over the timed steps."""
+    import synth
+    from paper_2104_11487_gb300 import SkipConvLayer
+    n, h, w, c, dy, dx = 1, 128, 128, 64, 1, 1
+    T = warmup + steps + 1
+    v = synth.round_to_bf16(synth.panning_video(6000, T, n, h, w, c, dy, dx))
+    frames = [torch.from_numpy(np.ascontiguousarray(v[t])).cuda().to(torch.bfloat16) for t in range(T)]
+    wts = torch.from_numpy(synth.he_weights(np.random.default_rng(6001), c, c, 3, bf16=True))
+    flow = torch.zeros((n, h, w, 2), dtype=torch.float32, device="cuda")
+    flow[..., 0], flow[..., 1] = float(dy), float(dx)
+    out = {"workload": "camera pan by (1, 1) px/frame over a 1 x 128x128x64 bf16 texture; 3x3 64->64, 8x8 blocks, "
+                       "eps 0.05, one-launch CUDA-core step; flow = the pan", "steps": steps}
+    for mode in ("plain", "warped"):
+        lay = SkipConvLayer(n, c, c, h, w, k=3, block=8, eps=0.05, dtype="bf16", conv_path=1, weights=wts)
+        step = (lambda x: lay.step(x)) if mode == "plain" else (lambda x: lay.step_warped(x, flow))
+        for t in range(warmup + 1):
+            step(frames[t])
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        torch.cuda.synchronize()
+        for i in range(steps):
+            flush_l2(flush)
+            ev[i][0].record(lay.stream)
+            step(frames[warmup + 1 + i])
+            ev[i][1].record(lay.stream)
+        torch.cuda.synchronize()
+        us = statistics.median(a.elapsed_time(b) for a, b in ev) * 1e3
+        lay.reset()
+        dens = []
+        for t in range(T):
+            step(frames[t])
+            if t > warmup:
+                dens.append(lay.gate()[2] / (n * lay.info.nby * lay.info.nbx))
+        out[mode] = {"us_per_step": us, "open_block_density": statistics.mean(dens)}
+        lay.close()
+    return out
+
+
 # ----------------------------------------------------------- CPU oracle
 def cpu_oracle_sample(seconds, density, max_frames=40):
     """The oracle as it stands, on the host cores: stream 0 of the same
@@ -599,10 +645,15 @@ def main():
 
     if args.workloads_only:
         flush = None if args.no_flush else torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-        rep = workloads_report(torch, flush, tc_peak, hbm, names=tuple(args.workloads_only.split(",")),
-                               link=args.link)
+        names = [x for x in args.workloads_only.split(",") if x]
+        out = {}
+        if "warped" in names:
+            names.remove("warped")
+            out["warped_residual"] = warped_report(torch, flush)
+        if names:
+            out["other_workloads"] = workloads_report(torch, flush, tc_peak, hbm, names=tuple(names), link=args.link)
         if rank == 0:
-            print(json.dumps({"other_workloads": rep}), flush=True)
+            print(json.dumps(out), flush=True)
         ranks.close()
         return 0
 
@@ -731,6 +782,9 @@ def main():
     # 5) the single-layer and stacked workloads
     if not args.no_workloads:
         line["other_workloads"] = workloads_report(torch, flush, tc_peak, hbm, link=args.link)
+
+    if not args.no_workloads:
+        line["warped_residual"] = warped_report(torch, flush)
 
     # 6) the CPU oracle on the host cores (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

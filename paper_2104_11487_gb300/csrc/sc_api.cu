@@ -139,7 +139,7 @@ static void free_buffers(Layer* L)
     prof_release(L);
     void* ptrs[] = {L->xbuf[0], L->xbuf[1], L->chg[0], L->chg[1], L->pix_l1, L->mask, L->list, L->counters,
                     L->z, L->y, L->bias, L->w_cc, L->w_tc, L->x_stage, L->sched, L->pnorm, L->gtag,
-                    L->pix_taps, L->gphi, L->w_loc, L->ychg, L->tile_chg, L->z_prev};
+                    L->pix_taps, L->gphi, L->w_loc, L->ychg, L->tile_chg, L->z_prev, L->tx};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     if (L->err_host) cudaFreeHost(L->err_host);

@@ -94,6 +94,8 @@ struct Layer {
     long long link_x_seen, link_sc_seen;
     long long steps;        // steps since create (never reset)
     float* z_prev;          // warped steps: copy of z before its warp (allocated at the first one)
+    float* tx;              // warped steps on the staged form: T(x_{t-1}) in fp32 (allocated at the first one)
+    CUtensorMap tmap_tx;    //   and its footprint boxes
 };
 
 // ------------------------------------------------------------------ launchers

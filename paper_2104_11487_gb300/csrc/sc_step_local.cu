@@ -47,6 +47,8 @@ using namespace ptx;
 
 constexpr int LT = 128;               // threads per CTA
 constexpr int LPI = 2;                // output locations per work item of the dense contraction
+constexpr int GIPT = 2;               // work items per thread and round (general form)
+constexpr int GKC = 16;               // contraction chunk staged in shared memory (general form)
 constexpr int MAX_TILE_BLOCKS = 16;   // sb <= 4
 
 struct LocalArgs {
@@ -322,69 +324,91 @@ __global__ void __launch_bounds__(LT) step_local_kernel(const LocalArgs a)
             if (y_here) y[zo] = from_f32<T>(activate(zv, a.act));
         }
     } else {
+        // rounds of up to IPT work items per thread; k in chunks of GKC whose weights (all output
+        // channels) and footprint offsets are staged in shared memory by the whole CTA
         const int nq = (a.opg + 3) >> 2;             // output-channel quads per group
         const int nm = (M + LPI - 1) / LPI;
         const int items = nm * a.groups * nq;
-        for (int it = threadIdx.x; it < items; it += LT) {
-            const int q = it % nq;
-            const int rest = it / nq;
-            const int grp = rest % a.groups, mi = rest / a.groups;
-            const int o = grp * a.opg + q * 4;
-            const int oend = grp * a.opg + a.opg;
-            int rb[LPI];
-            long long zl[LPI];
+        const int K = a.KH * a.KW * a.cpg;           // contraction length of one output channel
+        // [GKC][Co], 16-byte aligned for the quad loads
+        float* Wc = sm + (((size_t)FP * a.CP + FP + (size_t)span * span + 3) & ~(size_t)3);
+        int* toffs = reinterpret_cast<int*>(Wc + GKC * a.Co);      // [GKC] residual offset of k in the footprint
+        for (int it0 = 0; it0 < items; it0 += LT * GIPT) {
+            int o[GIPT], oend[GIPT], rb[GIPT][LPI];
+            long long zl[GIPT][LPI];
+            float acc[GIPT][LPI][4];
 #pragma unroll
-            for (int u = 0; u < LPI; ++u) {
-                const int m = mi * LPI + u;
-                if (m < M) {
-                    const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
-                    rb[u] = (li * a.stride * a.FW + lj * a.stride) * a.CP + grp * a.cpg;
-                    zl[u] = ((long long)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj;
-                } else {
-                    rb[u] = 0;
-                    zl[u] = -1;
+            for (int j = 0; j < GIPT; ++j) {
+                const int it = it0 + (int)threadIdx.x + j * LT;
+                const bool on = it < items;
+                const int q = on ? it % nq : 0;
+                const int rest = on ? it / nq : 0;
+                const int grp = rest % a.groups, mi = rest / a.groups;
+                o[j] = grp * a.opg + q * 4;
+                oend[j] = on ? grp * a.opg + a.opg : 0;   // 0: no work
+#pragma unroll
+                for (int u = 0; u < LPI; ++u) {
+                    const int m = mi * LPI + u;
+                    if (on && m < M) {
+                        const int loc = locs[m], li = loc >> 16, lj = loc & 0xffff;
+                        rb[j][u] = (li * a.stride * a.FW + lj * a.stride) * a.CP + grp * a.cpg;
+                        zl[j][u] = ((long long)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj;
+                    } else {
+                        rb[j][u] = 0;
+                        zl[j][u] = -1;
+                    }
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[j][u][e] = 0.f;
                 }
             }
-            float acc[LPI][4];
+            for (int k0 = 0; k0 < K; k0 += GKC) {
+                const int kc = min(GKC, K - k0);
+                __syncthreads();   // the previous chunk has been used
+                for (int e = threadIdx.x; e < kc * a.Co; e += LT) Wc[e] = __ldg(a.wcc + (size_t)k0 * a.Co + e);
+                if ((int)threadIdx.x < kc) {
+                    const int k = k0 + (int)threadIdx.x, tap = k / a.cpg, ci = k - tap * a.cpg;
+                    toffs[threadIdx.x] = ((tap / a.KW) * a.FW + tap % a.KW) * a.CP + ci;
+                }
+                __syncthreads();
+                for (int kk = 0; kk < kc; ++kk) {
+                    const int toff = toffs[kk];
+                    const float* wrow = Wc + kk * a.Co;
 #pragma unroll
-            for (int u = 0; u < LPI; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
-            for (int kh = 0; kh < a.KH; ++kh) {
-                for (int kw = 0; kw < a.KW; ++kw) {
-                    const float* wr = a.wcc + (size_t)((kh * a.KW + kw) * a.cpg) * a.Co + o;
-                    const int toff = (kh * a.FW + kw) * a.CP;
-#pragma unroll 4
-                    for (int ci = 0; ci < a.cpg; ++ci) {
+                    for (int j = 0; j < GIPT; ++j) {
+                        if (oend[j] == 0) continue;
                         float4 w;
                         if (V4) {
-                            w = __ldg(reinterpret_cast<const float4*>(wr + (size_t)ci * a.Co));
+                            w = *reinterpret_cast<const float4*>(wrow + o[j]);
                         } else {
-                            const float* wp = wr + (size_t)ci * a.Co;
-                            w.x = __ldg(wp);
-                            w.y = o + 1 < oend ? __ldg(wp + 1) : 0.f;
-                            w.z = o + 2 < oend ? __ldg(wp + 2) : 0.f;
-                            w.w = o + 3 < oend ? __ldg(wp + 3) : 0.f;
+                            w.x = wrow[o[j]];
+                            w.y = o[j] + 1 < oend[j] ? wrow[o[j] + 1] : 0.f;
+                            w.z = o[j] + 2 < oend[j] ? wrow[o[j] + 2] : 0.f;
+                            w.w = o[j] + 3 < oend[j] ? wrow[o[j] + 3] : 0.f;
                         }
 #pragma unroll
                         for (int u = 0; u < LPI; ++u) {
-                            const float r = R[rb[u] + toff + ci];
-                            acc[u][0] = fmaf(r, w.x, acc[u][0]);
-                            acc[u][1] = fmaf(r, w.y, acc[u][1]);
-                            acc[u][2] = fmaf(r, w.z, acc[u][2]);
-                            acc[u][3] = fmaf(r, w.w, acc[u][3]);
+                            const float r = R[rb[j][u] + toff];
+                            acc[j][u][0] = fmaf(r, w.x, acc[j][u][0]);
+                            acc[j][u][1] = fmaf(r, w.y, acc[j][u][1]);
+                            acc[j][u][2] = fmaf(r, w.z, acc[j][u][2]);
+                            acc[j][u][3] = fmaf(r, w.w, acc[j][u][3]);
                         }
                     }
                 }
             }
 #pragma unroll
-            for (int u = 0; u < LPI; ++u) {
-                if (zl[u] < 0) continue;
+            for (int j = 0; j < GIPT; ++j) {
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    if (o + j >= oend) continue;
-                    const size_t zo = (size_t)zl[u] * a.Co + o + j;
-                    const float zv = a.z[zo] + acc[u][j];
-                    a.z[zo] = zv;
-                    if (y_here) y[zo] = from_f32<T>(activate(zv, a.act));
+                for (int u = 0; u < LPI; ++u) {
+                    if (zl[j][u] < 0) continue;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        if (o[j] + e >= oend[j]) continue;
+                        const size_t zo = (size_t)zl[j][u] * a.Co + o[j] + e;
+                        const float zv = a.z[zo] + acc[j][u][e];
+                        a.z[zo] = zv;
+                        if (y_here) y[zo] = from_f32<T>(activate(zv, a.act));
+                    }
                 }
             }
         }
@@ -475,13 +499,38 @@ __device__ __forceinline__ int chunk_residual(const uint4& a, const uint4& b, fl
     return 4;
 }
 
+// x_t's chunk minus the matching fp32 values of the warped previous input.
+__device__ __forceinline__ int chunk_minus_f32(const uint4& a, const float* w, float (&r)[8], __nv_bfloat16*)
+{
+    const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+    const float4 w0 = reinterpret_cast<const float4*>(w)[0], w1 = reinterpret_cast<const float4*>(w)[1];
+    const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 fa = __bfloat1622float2(pa[k]);
+        r[2 * k] = fa.x - wv[2 * k];
+        r[2 * k + 1] = fa.y - wv[2 * k + 1];
+    }
+    return 8;
+}
+
+__device__ __forceinline__ int chunk_minus_f32(const uint4& a, const float* w, float (&r)[8], float*)
+{
+    const float4 w0 = reinterpret_cast<const float4*>(w)[0];
+    r[0] = __uint_as_float(a.x) - w0.x;
+    r[1] = __uint_as_float(a.y) - w0.y;
+    r[2] = __uint_as_float(a.z) - w0.z;
+    r[3] = __uint_as_float(a.w) - w0.w;
+    return 4;
+}
+
 __device__ __forceinline__ float2 load_pair(const float* p) { return *reinterpret_cast<const float2*>(p); }
 __device__ __forceinline__ float2 load_pair(const __nv_bfloat16* p)
 {
     return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
 }
 
-template <typename T, bool DW, int SW>
+template <typename T, bool DW, int SW, bool WP>
 __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_constant__ CUtensorMap tm_xt,
                                                                const __grid_constant__ CUtensorMap tm_xp,
                                                                const __grid_constant__ CUtensorMap tm_z,
@@ -497,6 +546,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
     uint8_t* base = align_smem_1024(smem_raw);
     const T* Xt = reinterpret_cast<const T*>(base);
     const T* Xp = reinterpret_cast<const T*>(base + a.off_xp);
+    const float* Xw = reinterpret_cast<const float*>(base + a.off_xp);   // WP: the warped previous input, fp32
     const T* Ws = reinterpret_cast<const T*>(base + a.off_w);
     float* R = reinterpret_cast<float*>(base + a.off_r);      // dense only: [FP][CP] residual
     float* P = reinterpret_cast<float*>(base + a.off_p);
@@ -579,7 +629,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         }
     }
     if (tid == 0) {
-        mbar_arrive_expect_tx(bar_x, 2u * (uint32_t)FP * (uint32_t)a.C * (uint32_t)sizeof(T));
+        mbar_arrive_expect_tx(bar_x, (uint32_t)FP * (uint32_t)a.C * (uint32_t)(sizeof(T) + (WP ? 4 : sizeof(T))));
         tma_load_4d(smem_u32(Xt), &tm_xt, bar_x, 0, fx0, fy0, nn);
         tma_load_4d(smem_u32(Xp), &tm_xp, bar_x, 0, fx0, fy0, nn);
         if (has_sc) {
@@ -617,15 +667,22 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         for (int it = tid; it < FP * CH; it += FT) {
             const int q = it / CH, k = it - (it / CH) * CH;
             const uint4 av = reinterpret_cast<const uint4*>(Xt + (size_t)q * a.C)[k];
-            const uint4 bv = reinterpret_cast<const uint4*>(Xp + (size_t)q * a.C)[k];
             float r[8];
-            const int ne = chunk_residual(av, bv, r, (T*)nullptr);
+            int ne;
+            if (WP) {
+                // r_t = x_t - T(x_{t-1}) (Eq. 10-11); the commit compared the raw frames in the pre-pass
+                ne = chunk_minus_f32(av, Xw + (size_t)q * a.C + k * EPC, r, (T*)nullptr);
+                Dp[it] = 0;
+            } else {
+                const uint4 bv = reinterpret_cast<const uint4*>(Xp + (size_t)q * a.C)[k];
+                ne = chunk_residual(av, bv, r, (T*)nullptr);
+                Dp[it] = ((av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w)) != 0u;
+            }
             float sum = 0.f;
 #pragma unroll
             for (int e = 0; e < 8; ++e)
                 if (e < ne) sum += fabsf(r[e]);
             Pp[it] = sum;
-            Dp[it] = ((av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w)) != 0u;
             if (!DW) {
                 float4* rr = reinterpret_cast<float4*>(R + (size_t)q * a.CP + k * EPC);
                 rr[0] = make_float4(r[0], r[1], r[2], r[3]);
@@ -648,8 +705,8 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
     __syncthreads();
 
     // slice 0: the commit of x_t for the owned pixels (one thread per pixel and chunk inside the
-    // footprint, a warp per pixel outside it), and the pixels' change flags
-    if (sl == 0) {
+    // footprint, a warp per pixel outside it), and the pixels' change flags (WP: done by the pre-pass)
+    if (sl == 0 && !WP) {
         for (int it = tid; it < npx * CH; it += FT) {
             const int q = it / CH, k = it - (it / CH) * CH;
             const int iy = own_y0 + q / oww, ix = own_x0 + q % oww;
@@ -778,7 +835,8 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
 #pragma unroll
                         for (int kw = 0; kw < 3; ++kw) {
                             const size_t e = (size_t)(p0 + kh * a.FW + kw) * a.C + c;
-                            const float2 xa = load_pair(Xt + e), xb = load_pair(Xp + e);
+                            const float2 xa = load_pair(Xt + e);
+                            const float2 xb = WP ? *reinterpret_cast<const float2*>(Xw + e) : load_pair(Xp + e);
                             acc0 = fmaf(wreg[kh * 3 + kw].x, xa.x - xb.x, acc0);
                             acc1 = fmaf(wreg[kh * 3 + kw].y, xa.y - xb.y, acc1);
                         }
@@ -786,7 +844,8 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
                     for (int kh = 0; kh < a.KH; ++kh)
                         for (int kw = 0; kw < a.KW; ++kw) {
                             const size_t e = (size_t)(p0 + kh * a.FW + kw) * a.C + c;
-                            const float2 xa = load_pair(Xt + e), xb = load_pair(Xp + e);
+                            const float2 xa = load_pair(Xt + e);
+                            const float2 xb = WP ? *reinterpret_cast<const float2*>(Xw + e) : load_pair(Xp + e);
                             const float2 w = load_pair(Ws + (kh * a.KW + kw) * a.C + c);
                             acc0 = fmaf(w.x, xa.x - xb.x, acc0);
                             acc1 = fmaf(w.y, xa.y - xb.y, acc1);
@@ -957,7 +1016,8 @@ LocalShape local_shape(const Layer& L, int sb)
     s.FW = (s.span - 1) * L.p.stride + L.p.k_w;
     s.CP = L.p.c_in | 1;   // odd pixel stride: neighbouring locations fall in different banks
     const size_t fp = (size_t)s.FH * s.FW;
-    s.smem = (fp * s.CP + fp + (size_t)s.span * s.span) * sizeof(float);
+    // residual, norms, location table, and the dense contraction's weight chunk and offsets
+    s.smem = (fp * s.CP + fp + (size_t)s.span * s.span + 3 + (size_t)GKC * L.p.c_out + GKC) * sizeof(float);
     return s;
 }
 
@@ -998,7 +1058,7 @@ inline uint32_t up128(size_t v) { return (uint32_t)((v + 127) & ~(size_t)127); }
 
 bool is_depthwise(const Layer& L) { return L.cpg == 1 && L.opg == 1; }
 
-StagedShape staged_shape(const Layer& L, int sb)
+StagedShape staged_shape(const Layer& L, int sb, bool wp = false)
 {
     StagedShape t;
     t.g = local_shape(L, sb);
@@ -1020,8 +1080,10 @@ StagedShape staged_shape(const Layer& L, int sb)
     t.own_max = (size_t)std::max(own_h, 0) * std::max(own_w, 0);
     const size_t tile_elems = (size_t)t.g.span * t.g.span * t.zw;
     const uint32_t xb = up128(fp * L.p.c_in * L.esize);
+    // the previous input's footprint: x_{t-1} in the dtype, or (wp) its warp T(x_{t-1}) in fp32
+    const uint32_t pb = wp ? up128(fp * L.p.c_in * sizeof(float)) : xb;
     t.off_xp = xb;
-    t.off_w = 2 * xb;
+    t.off_w = xb + pb;
     t.off_r = t.off_w + up128(t.wbytes);
     t.off_p = t.off_r + (dw ? 0 : up128(fp * t.g.CP * sizeof(float)));
     t.off_loc = t.off_p + up128(fp * sizeof(float));
@@ -1041,14 +1103,14 @@ StagedShape staged_shape(const Layer& L, int sb)
 // multiple of 16 bytes, every box edge at most 256), of the z tile (c_out a
 // multiple of 4) and of the shortcut tile (c_out a multiple of 16 bytes of
 // the dtype), and a dense (groups = 1) or depthwise layer.
-bool staged_ok(const Layer& L, StagedShape* out)
+bool staged_ok(const Layer& L, StagedShape* out, bool wp = false)
 {
     if (!(L.p.groups == 1 || is_depthwise(L))) return false;
     if ((L.p.c_in * L.esize) % 16 || L.p.c_in > 256) return false;
     if (L.p.c_out % 4 || (L.p.emit_y && (L.p.c_out * L.esize) % 16)) return false;
     int sb = L.p.block >= 4 ? 1 : (4 + L.p.block - 1) / L.p.block;
-    StagedShape t = staged_shape(L, sb);
-    while (t.smem > LOCAL_MAX_SMEM && sb > 1) t = staged_shape(L, --sb);
+    StagedShape t = staged_shape(L, sb, wp);
+    while (t.smem > LOCAL_MAX_SMEM && sb > 1) t = staged_shape(L, --sb, wp);
     if (t.smem > LOCAL_MAX_SMEM || t.g.FH > 256 || t.g.FW > 256 || t.g.span > 256 || t.zw > 256) return false;
     if ((long long)L.p.n_streams * ((L.nby + sb - 1) / sb) * ((L.nbx + sb - 1) / sb) * t.nsl > 0x7fffffffLL)
         return false;
@@ -1089,17 +1151,47 @@ bool encode_tile_map(CUtensorMap* m, const void* base, const Layer& L, const Sta
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <typename T>
+template <typename T, bool WP>
 const void* staged_kernel_of(const Layer& L, int sw)
 {
-    if (is_depthwise(L)) return (const void*)step_local_staged_kernel<T, true, SW_WIDE>;
-    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<T, false, SW_NARROW>
-                           : (const void*)step_local_staged_kernel<T, false, SW_WIDE>;
+    if (is_depthwise(L)) return (const void*)step_local_staged_kernel<T, true, SW_WIDE, WP>;
+    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<T, false, SW_NARROW, WP>
+                           : (const void*)step_local_staged_kernel<T, false, SW_WIDE, WP>;
 }
 
-const void* staged_kernel_of(const Layer& L, int sw)
+const void* staged_kernel_of(const Layer& L, int sw, bool wp = false)
 {
-    return L.p.dtype == SKIPCONV_BF16 ? staged_kernel_of<__nv_bfloat16>(L, sw) : staged_kernel_of<float>(L, sw);
+    if (L.p.dtype == SKIPCONV_BF16)
+        return wp ? staged_kernel_of<__nv_bfloat16, true>(L, sw) : staged_kernel_of<__nv_bfloat16, false>(L, sw);
+    return wp ? staged_kernel_of<float, true>(L, sw) : staged_kernel_of<float, false>(L, sw);
+}
+
+// Warped residual (Eq. 10-11), input side, before the staged kernel: T(x_{t-1})
+// into an fp32 frame (a warp per pixel, lanes over channels), and the commit of
+// x_t with the pixels' change flags, which compare the raw frames.
+template <typename T>
+__global__ void __launch_bounds__(256) warp_prev_kernel(const T* __restrict__ xt, const T* __restrict__ xp,
+                                                        T* __restrict__ xn, const uint8_t* __restrict__ chg_prev,
+                                                        uint8_t* __restrict__ chg_cur, const float* __restrict__ flow,
+                                                        float* __restrict__ tx, int n, int H, int W, int C)
+{
+    const int lane = threadIdx.x & 31;
+    const long long npx = (long long)n * H * W;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    for (long long pix = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; pix < npx; pix += nwarps) {
+        const int ix = (int)(pix % W), iy = (int)((pix / W) % H), nn = (int)(pix / ((long long)W * H));
+        const Bilinear bl = bilinear_of(flow, nn, H, W, C, iy, ix);
+        const size_t base = (size_t)pix * C;
+        unsigned d = 0;
+        for (int c = lane; c < C; c += 32) {
+            tx[base + c] = warped_at(xp, bl, c);
+            d |= bits_of(xt[base + c]) ^ bits_of(xp[base + c]);
+        }
+        const bool changed = __any_sync(0xffffffffu, d != 0);
+        if (changed || chg_prev[pix])
+            for (int c = lane; c < C; c += 32) xn[base + c] = xt[base + c];
+        if (lane == 0) chg_cur[pix] = changed ? 1 : 0;
+    }
 }
 
 cudaLaunchConfig_t pdl_config(const Layer& L, long long grid, int threads, size_t smem, cudaLaunchAttribute* attr)
@@ -1114,6 +1206,64 @@ cudaLaunchConfig_t pdl_config(const Layer& L, long long grid, int threads, size_
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cfg;
+}
+
+// The staged form's launch: tm_prev maps the previous input's footprints (x_{t-1}; for a warped
+// step T(x_{t-1}) in fp32, wp = true).
+cudaError_t launch_staged(Layer& L, const StagedShape& t, const void* x_t, const void* shortcut, int force,
+                          const Layer* px, const Layer* psc, const CUtensorMap* tm_prev, bool wp)
+{
+    const int cur = (int)(L.t & 1), nxt = cur ^ 1;
+    cudaLaunchAttribute attr[1];
+    alignas(64) CUtensorMap tm_xt;
+    if (!encode_footprint_map(&tm_xt, x_t, L, t)) {
+        set_error("tensor map of x_t rejected");
+        return cudaErrorInvalidValue;
+    }
+    FastArgs a;
+    a.wpack = L.w_loc;
+    a.wbytes = t.wbytes;
+    a.xt = x_t;
+    a.xp = L.xbuf[cur];
+    a.xn = L.xbuf[nxt];
+    a.chg_prev = L.chg[nxt];
+    a.chg_cur = L.chg[cur];
+    a.z = L.z;
+    a.y = L.y;
+    a.sc = L.y ? shortcut : nullptr;
+    a.mask = L.mask;
+    a.list = L.list;
+    a.count_cur = step_count(L);
+    a.count_next = next_count(L);
+    a.err = L.err_dev;
+    a.force = force;
+    a.n = L.p.n_streams; a.H = L.p.h; a.W = L.p.w; a.C = L.p.c_in; a.Ho = L.ho; a.Wo = L.wo;
+    a.Co = L.p.c_out; a.KH = L.p.k_h; a.KW = L.p.k_w; a.stride = L.p.stride; a.pad = L.p.pad; a.b = L.p.block;
+    a.nby = L.nby; a.nbx = L.nbx; a.act = L.p.activation;
+    a.sb = t.g.sb;
+    a.nty = (L.nby + t.g.sb - 1) / t.g.sb;
+    a.ntx = (L.nbx + t.g.sb - 1) / t.g.sb;
+    a.FH = t.g.FH; a.FW = t.g.FW; a.CP = t.g.CP; a.nsl = t.nsl; a.K = L.p.k_h * L.p.k_w * L.p.c_in;
+    a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
+    a.off_scr = t.off_scr; a.off_z = t.off_z; a.off_sc = t.off_sc; a.off_chg = t.off_chg; a.off_dq = t.off_dq;
+    a.thr = L.gate_thr;
+    a.px_chg = px ? px->ychg : nullptr;
+    a.pxb = px ? px->p.block : 1; a.pxnby = px ? px->nby : 1; a.pxnbx = px ? px->nbx : 1;
+    a.psc_chg = psc ? psc->ychg : nullptr;
+    a.pscb = psc ? psc->p.block : 1; a.pscnby = psc ? psc->nby : 1; a.pscnbx = psc ? psc->nbx : 1;
+    a.ychg = L.ychg;
+    a.tile_chg_prev = L.tile_chg + (size_t)nxt * L.ntiles;
+    a.tile_chg_cur = L.tile_chg + (size_t)cur * L.ntiles;
+    alignas(64) CUtensorMap tm_sc = L.tmap_ztile;   // unused without a shortcut
+    if (a.sc && !encode_tile_map(&tm_sc, a.sc, L, t, false)) {
+        set_error("tensor map of the shortcut rejected");
+        return cudaErrorInvalidValue;
+    }
+    const long long grid = (long long)a.n * a.nty * a.ntx * t.nsl;
+    cudaLaunchConfig_t cfg = pdl_config(L, grid, FT, t.smem, attr);
+    CUtensorMap* tm_z = const_cast<CUtensorMap*>(&L.tmap_ztile);
+    void* args[] = {&tm_xt, const_cast<CUtensorMap*>(tm_prev), tm_z, &tm_sc, &a};
+    return cudaLaunchKernelExC(&cfg, staged_kernel_of(L, t.sw, wp), args);
 }
 
 }  // namespace
@@ -1195,7 +1345,9 @@ cudaError_t step_local_prepare(Layer& L)
         e = cudaMemsetAsync(L.tile_chg, 0, 2 * (size_t)L.ntiles, L.stream);
         if (e == cudaSuccess) e = alloc_ychg(L);
         if (e == cudaSuccess) e = ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
-        // warped steps run the general form
+        // warped steps run the staged form's warped variant, or the general form when it does not fit
+        StagedShape tw;
+        if (e == cudaSuccess && staged_ok(L, &tw, true)) e = ensure_dynamic_smem(staged_kernel_of(L, tw.sw, true), tw.smem);
         if (e == cudaSuccess && choose_shape(L).smem <= LOCAL_MAX_SMEM) e = ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
         return e;
     }
@@ -1210,59 +1362,49 @@ cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, i
 {
     const int cur = (int)(L.t & 1), nxt = cur ^ 1;
     cudaLaunchAttribute attr[1];
-    if (L.local_staged && !flow) {   // warped residuals take the general form (its loads sample the warp)
-        StagedShape t;
+    StagedShape t;
+    if (flow && L.local_staged && staged_ok(L, &t, true)) {
+        // warped residual on the staged form: T(x_{t-1}) and the commit first, then the step with the
+        // warped frame as its previous input
+        const size_t nx = (size_t)L.p.n_streams * L.p.h * L.p.w * L.p.c_in;
+        if (!L.tx) {
+            cudaError_t e = cudaMalloc((void**)&L.tx, nx * sizeof(float));
+            if (e != cudaSuccess) {
+                L.tx = nullptr;
+                return e;
+            }
+            L.state_bytes += nx * sizeof(float);
+            EncodeTiledFn enc = encode_tiled_fn();
+            const cuuint64_t C = L.p.c_in, W = L.p.w, H = L.p.h, N = L.p.n_streams;
+            cuuint64_t dims[4] = {C, W, H, N};
+            cuuint64_t strides[3] = {C * 4, W * C * 4, H * W * C * 4};
+            cuuint32_t box[4] = {(cuuint32_t)C, (cuuint32_t)t.g.FW, (cuuint32_t)t.g.FH, 1};
+            cuuint32_t estr[4] = {1, 1, 1, 1};
+            if (!enc || enc(&L.tmap_tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, L.tx, dims, strides, box, estr,
+                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+                set_error("tensor map of the warped frame rejected");
+                return cudaErrorInvalidValue;
+            }
+        }
+        const long long npx = (long long)L.p.n_streams * L.p.h * L.p.w;
+        const long long blocks = (npx + 7) / 8, cap = (long long)L.num_sms * 16;
+        const int grid = (int)(blocks < cap ? blocks : cap);
+        if (L.p.dtype == SKIPCONV_BF16)
+            warp_prev_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(
+                (const __nv_bfloat16*)x_t, (const __nv_bfloat16*)L.xbuf[cur], (__nv_bfloat16*)L.xbuf[nxt], L.chg[nxt],
+                L.chg[cur], flow, L.tx, L.p.n_streams, L.p.h, L.p.w, L.p.c_in);
+        else
+            warp_prev_kernel<float><<<grid, 256, 0, L.stream>>>((const float*)x_t, (const float*)L.xbuf[cur],
+                                                                (float*)L.xbuf[nxt], L.chg[nxt], L.chg[cur], flow,
+                                                                L.tx, L.p.n_streams, L.p.h, L.p.w, L.p.c_in);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        return launch_staged(L, t, x_t, shortcut, force, nullptr, nullptr, &L.tmap_tx, true);
+    }
+    if (L.local_staged && !flow) {
         if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
-        alignas(64) CUtensorMap tm_xt;
-        if (!encode_footprint_map(&tm_xt, x_t, L, t)) {
-            set_error("tensor map of x_t rejected");
-            return cudaErrorInvalidValue;
-        }
-        FastArgs a;
-        a.wpack = L.w_loc;
-        a.wbytes = t.wbytes;
-        a.xt = x_t;
-        a.xp = L.xbuf[cur];
-        a.xn = L.xbuf[nxt];
-        a.chg_prev = L.chg[nxt];
-        a.chg_cur = L.chg[cur];
-        a.z = L.z;
-        a.y = L.y;
-        a.sc = L.y ? shortcut : nullptr;
-        a.mask = L.mask;
-        a.list = L.list;
-        a.count_cur = step_count(L);
-        a.count_next = next_count(L);
-        a.err = L.err_dev;
-        a.force = force;
-        a.n = L.p.n_streams; a.H = L.p.h; a.W = L.p.w; a.C = L.p.c_in; a.Ho = L.ho; a.Wo = L.wo;
-        a.Co = L.p.c_out; a.KH = L.p.k_h; a.KW = L.p.k_w; a.stride = L.p.stride; a.pad = L.p.pad; a.b = L.p.block;
-        a.nby = L.nby; a.nbx = L.nbx; a.act = L.p.activation;
-        a.sb = t.g.sb;
-        a.nty = (L.nby + t.g.sb - 1) / t.g.sb;
-        a.ntx = (L.nbx + t.g.sb - 1) / t.g.sb;
-        a.FH = t.g.FH; a.FW = t.g.FW; a.CP = t.g.CP; a.nsl = t.nsl; a.K = L.p.k_h * L.p.k_w * L.p.c_in;
-        a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
-        a.off_scr = t.off_scr; a.off_z = t.off_z; a.off_sc = t.off_sc; a.off_chg = t.off_chg; a.off_dq = t.off_dq;
-        a.thr = L.gate_thr;
-        a.px_chg = px ? px->ychg : nullptr;
-        a.pxb = px ? px->p.block : 1; a.pxnby = px ? px->nby : 1; a.pxnbx = px ? px->nbx : 1;
-        a.psc_chg = psc ? psc->ychg : nullptr;
-        a.pscb = psc ? psc->p.block : 1; a.pscnby = psc ? psc->nby : 1; a.pscnbx = psc ? psc->nbx : 1;
-        a.ychg = L.ychg;
-        a.tile_chg_prev = L.tile_chg + (size_t)nxt * L.ntiles;
-        a.tile_chg_cur = L.tile_chg + (size_t)cur * L.ntiles;
-        alignas(64) CUtensorMap tm_sc = L.tmap_ztile;   // unused without a shortcut
-        if (a.sc && !encode_tile_map(&tm_sc, a.sc, L, t, false)) {
-            set_error("tensor map of the shortcut rejected");
-            return cudaErrorInvalidValue;
-        }
-        const long long grid = (long long)a.n * a.nty * a.ntx * t.nsl;
-        cudaLaunchConfig_t cfg = pdl_config(L, grid, FT, t.smem, attr);
-        const CUtensorMap* tm_xp = &L.tmap_fp[cur];
-        CUtensorMap* tm_z = const_cast<CUtensorMap*>(&L.tmap_ztile);
-        void* args[] = {&tm_xt, const_cast<CUtensorMap*>(tm_xp), tm_z, &tm_sc, &a};
-        return cudaLaunchKernelExC(&cfg, staged_kernel_of(L, t.sw), args);
+        return launch_staged(L, t, x_t, shortcut, force, px, psc, &L.tmap_fp[cur], false);
     }
     const LocalShape s = choose_shape(L);
     LocalArgs a;

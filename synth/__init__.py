@@ -11,6 +11,7 @@ from .video import (  # noqa: F401
     round_to_bf16,
     moving_squares_video,
     moving_rect_video,
+    panning_video,
     traffic_video,
     block_perturbation_video,
     he_weights,

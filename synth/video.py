@@ -83,6 +83,23 @@ def moving_squares_video(seed: int, T: int, h: int, w: int, c: int, n_squares: i
     return out
 
 
+def panning_video(seed: int, T: int, n: int, h: int, w: int, c: int, dy: int, dx: int) -> np.ndarray:
+    """A camera pan: frame t of stream s is the h x w window of a seeded
+    U[0,1) texture whose top-left corner is at (t * dy, t * dx) (plus a
+    margin so the window stays inside), i.e. frame t at pixel p equals frame
+    t-1 at p + (dy, dx).  [T, n, h, w, c] float32."""
+    rng = np.random.default_rng(seed)
+    H, Wd = h + T * abs(dy) + 1, w + T * abs(dx) + 1
+    oy, ox = (T * abs(dy) if dy < 0 else 0), (T * abs(dx) if dx < 0 else 0)
+    out = np.empty((T, n, h, w, c), np.float32)
+    for s in range(n):
+        tex = rng.random((H, Wd, c), dtype=np.float32)
+        for t in range(T):
+            y0, x0 = oy + t * dy, ox + t * dx
+            out[t, s] = tex[y0:y0 + h, x0:x0 + w]
+    return out
+
+
 def moving_rect_video(seed: int, T: int, h: int, w: int, c: int, n_rects: int, rh: int, rw: int,
                       speed: int = 2, jitter: int = 1) -> np.ndarray:
     """Static background plus textured rh x rw rectangles moving `speed`
