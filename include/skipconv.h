@@ -234,10 +234,11 @@ SKIPCONV_API int skipconv_check_device(skipconv_handle h);
  * state commit), 1 gate_block (support norm, block gate, compaction), 2 the
  * convolution of the open blocks (either path), 3 y refresh, 4 the fused
  * tensor-core step (all of 0-2 in one launch), 5 the one-launch CUDA-core step
- * (all of 0-3).  Launch counts are always kept; with enable = 1
+ * (all of 0-3), 6 the warp pass of skipconv_step_warped (z~ and, on the staged
+ * form, x_{t-1}, Eq. 10-11).  Launch counts are always kept; with enable = 1
  * each launch is also bracketed by CUDA events on the handle's stream.
  * skipconv_profile resets both. */
-#define SKIPCONV_PROFILE_KINDS 6
+#define SKIPCONV_PROFILE_KINDS 7
 SKIPCONV_API int skipconv_profile(skipconv_handle h, int enable);
 /* Synchronise the stream and report, per kernel kind (arrays of
  * SKIPCONV_PROFILE_KINDS), the launches and the summed event-timed

@@ -20,7 +20,7 @@ GATE_INPUT_MEAN, GATE_INPUT_SUM, GATE_OUTPUT, GATE_GUMBEL = 0, 1, 2, 3
 F32, BF16 = 0, 1
 ACT_NONE, ACT_RELU, ACT_SILU = 0, 1, 2
 PATH_AUTO, PATH_CUDA_CORE, PATH_TENSOR_CORE, PATH_TENSOR_CORE_SEPARATE, PATH_CUDA_CORE_SEPARATE = 0, 1, 2, 3, 4
-PROFILE_KINDS = 6   # gate_pixel, gate_block, conv, y_refresh, fused tensor-core step, CUDA-core step
+PROFILE_KINDS = 7   # gate_pixel, gate_block, conv, y_refresh, fused tensor-core step, CUDA-core step, warp pass
 
 # Every function the header declares, with its ctypes signature.
 SIGNATURES = {

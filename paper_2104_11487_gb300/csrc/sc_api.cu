@@ -519,21 +519,10 @@ int skipconv_step_warped(skipconv_handle h, const void* x_t, const void* shortcu
     }
     // a key frame has no previous frame to warp: it is the plain key-frame step
     if (L->key) return skipconv_step(h, x_t, shortcut);
-    const size_t nz = (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out;
-    cudaError_t e = cudaSuccess;
-    if (!L->z_prev) {
-        e = cudaMalloc((void**)&L->z_prev, nz * sizeof(float));
-        if (e != cudaSuccess) {
-            L->z_prev = nullptr;
-            return status_of(e);
-        }
-        L->state_bytes += nz * sizeof(float);
-    }
     const int cur = (int)(L->t & 1);
     // z~_t = T~(z~_{t-1}) everywhere, then + w * r_t at the open blocks with r_t = x_t - T(x_{t-1})
-    int slot = prof_begin(L, 3);
-    e = cudaMemcpyAsync(L->z_prev, L->z, nz * sizeof(float), cudaMemcpyDeviceToDevice, L->stream);
-    if (e == cudaSuccess) e = launch_warp_z(*L, L->z_prev, flow, L->y != nullptr && !shortcut);
+    int slot = prof_begin(L, 6);
+    cudaError_t e = launch_step_warp_pass(*L, x_t, shortcut, flow);
     prof_end(L, slot);
     if (e == cudaSuccess) {
         slot = prof_begin(L, 5);

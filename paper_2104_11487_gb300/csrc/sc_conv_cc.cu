@@ -12,7 +12,6 @@
 //   y_refresh  : y = act(z + shortcut) over the whole frame (layer output handed
 //                to the next layer; z itself stays pre-activation, Sec. 3.1).
 //   reset_z    : z = bias (state after a reset).
-//   warp_z     : z = T~(z) for a warped residual (Eq. 10-11).
 //   pack       : weight repacking at create, and ||w||_1 for the Output-Norm gate.
 #include "sc_internal.h"
 
@@ -199,36 +198,6 @@ __global__ void y_refresh_kernel(const float* __restrict__ z, const T* __restric
     }
 }
 
-// Warped residual (Eq. 10-11), output side: z_dst = T~(z_src), the previous
-// output sampled at (i + dy, j + dx) by bilinear interpolation of the four
-// surrounding locations (zero outside), with the input's flow (the layer
-// keeps the frame size); y = act(z_dst) too when y is kept without a shortcut.
-template <typename T>
-__global__ void warp_z_kernel(const float* __restrict__ zsrc, float* __restrict__ zdst, const float* __restrict__ flow,
-                              T* __restrict__ y, int act, int n, int H, int W, int C)
-{
-    const long long count = (long long)n * H * W * C;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < count;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int c = (int)(i % C);
-        const long long pix = i / C;
-        const int x = (int)(pix % W), yy = (int)((pix / W) % H), nn = (int)(pix / ((long long)W * H));
-        const float sy = (float)yy + flow[2 * pix], sx = (float)x + flow[2 * pix + 1];
-        const float y0f = floorf(sy), x0f = floorf(sx);
-        const float ay = sy - y0f, ax = sx - x0f;
-        const int y0 = (int)y0f, x0 = (int)x0f;
-        const int ys[4] = {y0, y0, y0 + 1, y0 + 1}, xs[4] = {x0, x0 + 1, x0, x0 + 1};
-        const float w[4] = {(1.f - ay) * (1.f - ax), (1.f - ay) * ax, ay * (1.f - ax), ay * ax};
-        float v = 0.f;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-            if (ys[q] >= 0 && ys[q] < H && xs[q] >= 0 && xs[q] < W)
-                v += w[q] * zsrc[(((size_t)nn * H + ys[q]) * W + xs[q]) * C + c];
-        zdst[i] = v;
-        if (y) y[i] = from_f32<T>(activate(v, act));
-    }
-}
-
 __global__ void reset_z_kernel(float* __restrict__ z, const float* __restrict__ bias, long long count, int co)
 {
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < count;
@@ -311,22 +280,6 @@ cudaError_t launch_y_refresh(const Layer& L, const void* shortcut)
     else
         y_refresh_kernel<float><<<grid, 256, 0, L.stream>>>(L.z, (const float*)shortcut, (float*)L.y, count,
                                                            L.p.activation);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_warp_z(const Layer& L, const float* zsrc, const float* flow, bool write_y)
-{
-    const long long count = (long long)L.p.n_streams * L.ho * L.wo * L.p.c_out;
-    long long blocks = (count + 255) / 256;
-    const long long cap = (long long)L.num_sms * 8;
-    const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
-    if (L.p.dtype == SKIPCONV_BF16)
-        warp_z_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(zsrc, L.z, flow,
-                                                                write_y ? (__nv_bfloat16*)L.y : nullptr,
-                                                                L.p.activation, L.p.n_streams, L.ho, L.wo, L.p.c_out);
-    else
-        warp_z_kernel<float><<<grid, 256, 0, L.stream>>>(zsrc, L.z, flow, write_y ? (float*)L.y : nullptr,
-                                                        L.p.activation, L.p.n_streams, L.ho, L.wo, L.p.c_out);
     return cudaGetLastError();
 }
 

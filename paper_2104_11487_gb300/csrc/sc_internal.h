@@ -93,7 +93,7 @@ struct Layer {
     struct Layer* link_sc;
     long long link_x_seen, link_sc_seen;
     long long steps;        // steps since create (never reset)
-    float* z_prev;          // warped steps: copy of z before its warp (allocated at the first one)
+    float* z_prev;          // warped steps: the second z buffer (the warp writes it, then the two swap)
     float* tx;              // warped steps on the staged form: T(x_{t-1}) in fp32 (allocated at the first one)
     CUtensorMap tmap_tx;    //   and its footprint boxes
 };
@@ -119,8 +119,6 @@ cudaError_t launch_gate_blocks_gumbel(const Layer& L, int force);
 cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
 cudaError_t launch_y_refresh(const Layer& L, const void* shortcut);
 cudaError_t launch_reset_z(const Layer& L);
-// z = T~(zsrc) (bilinear warp with the input's flow, Eq. 10-11), and y = act(z) when write_y
-cudaError_t launch_warp_z(const Layer& L, const float* zsrc, const float* flow, bool write_y);
 cudaError_t launch_pack_weights(Layer& L, const void* w_oihw, double* w_l1_out);
 
 // Tensor-core convolution (sc_conv_tc.cu)
@@ -149,13 +147,18 @@ constexpr size_t LOCAL_MAX_SMEM = 226 * 1024;
 constexpr double LOCAL_AUTO_MAX_MACS = 67108864.0;   // 2^26
 bool step_local_preferred(const Layer& L);
 bool step_local_supported(const Layer& L);
-// Warped residuals (Eq. 10-11) run on this step's general form: the layer must keep the frame size.
+// Warped residuals (Eq. 10-11) run on this step (the staged form's warped variant, else the general
+// form): the layer must keep the frame size.
 bool step_local_warp_supported(const Layer& L);
 cudaError_t step_local_prepare(Layer& L);
 // px / psc: the linked producers of x_t / of the shortcut whose y-change flags
 // are valid for this step (NULL: not linked, or not valid for this step).
 cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, int force, const Layer* px,
                               const Layer* psc, const float* flow = nullptr);
+// Warped residual (Eq. 10-11), before launch_step_local with the same flow: warps z~ into the second z
+// buffer, which becomes z (y = act of it without a shortcut), and, where the staged form's warped
+// variant runs, writes T(x_{t-1}) in fp32 and commits x_t with the change flags.
+cudaError_t launch_step_warp_pass(Layer& L, const void* x_t, const void* shortcut, const float* flow);
 
 // Driver entry point for tensor-map encoding (resolved once through the runtime).
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

@@ -1166,31 +1166,144 @@ const void* staged_kernel_of(const Layer& L, int sw, bool wp = false)
     return wp ? staged_kernel_of<float, true>(L, sw) : staged_kernel_of<float, false>(L, sw);
 }
 
-// Warped residual (Eq. 10-11), input side, before the staged kernel: T(x_{t-1})
-// into an fp32 frame (a warp per pixel, lanes over channels), and the commit of
-// x_t with the pixels' change flags, which compare the raw frames.
-template <typename T>
-__global__ void __launch_bounds__(256) warp_prev_kernel(const T* __restrict__ xt, const T* __restrict__ xp,
-                                                        T* __restrict__ xn, const uint8_t* __restrict__ chg_prev,
-                                                        uint8_t* __restrict__ chg_cur, const float* __restrict__ flow,
-                                                        float* __restrict__ tx, int n, int H, int W, int C)
+// The staged form's warped variant runs where it tiles the frame, slices the
+// channels and packs the weights as the plain form does (the z tile map, the
+// per-tile flags and the packed weights are the plain form's).
+bool staged_wp_ok(const Layer& L, StagedShape* t, StagedShape* tw)
 {
-    const int lane = threadIdx.x & 31;
-    const long long npx = (long long)n * H * W;
-    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
-    for (long long pix = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; pix < npx; pix += nwarps) {
-        const int ix = (int)(pix % W), iy = (int)((pix / W) % H), nn = (int)(pix / ((long long)W * H));
-        const Bilinear bl = bilinear_of(flow, nn, H, W, C, iy, ix);
-        const size_t base = (size_t)pix * C;
-        unsigned d = 0;
-        for (int c = lane; c < C; c += 32) {
-            tx[base + c] = warped_at(xp, bl, c);
-            d |= bits_of(xt[base + c]) ^ bits_of(xp[base + c]);
+    if (!L.local_staged || !staged_ok(L, t) || !staged_ok(L, tw, true)) return false;
+    return tw->g.sb == t->g.sb && tw->g.span == t->g.span && tw->g.FH == t->g.FH && tw->g.FW == t->g.FW &&
+           tw->zw == t->zw && tw->sw == t->sw && tw->nsl == t->nsl && tw->wbytes == t->wbytes;
+}
+
+// Warped residual (Eq. 10-11), before the step, in one pass over the frame with
+// the bilinear weights taken once per pixel:
+//   - the output state's warp z~ <- T~(z~_{t-1}) from zsrc into zdst (the layer
+//     keeps the frame size, so T~ uses the same flow), and y = act of it when y
+//     is given (a step without a shortcut refreshes y only at open blocks);
+//   - for the staged form (tx != NULL), T(x_{t-1}) into an fp32 frame, and the
+//     commit of x_t with the pixels' change flags, which compare the raw frames.
+// A group of 2^lp_log2 lanes per pixel, 16-byte vectors of channels.
+struct WarpPreArgs {
+    const float* flow;
+    const float* zsrc;
+    float* zdst;
+    void* y;
+    const void* xt;
+    const void* xp;
+    void* xn;
+    const uint8_t* chg_prev;
+    uint8_t* chg_cur;
+    float* tx;
+    int n, H, W, C, Co, act, lp_log2;
+};
+
+__device__ __forceinline__ void unpack16(const uint4& v, float (&f)[8], const float*)
+{
+    f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y); f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+}
+__device__ __forceinline__ void unpack16(const uint4& v, float (&f)[8], const __nv_bfloat16*)
+{
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 t = __bfloat1622float2(h[k]);
+        f[2 * k] = t.x;
+        f[2 * k + 1] = t.y;
+    }
+}
+__device__ __forceinline__ void store_act4(float* y, const float4& v, int act)
+{
+    *reinterpret_cast<float4*>(y) = make_float4(activate(v.x, act), activate(v.y, act), activate(v.z, act), activate(v.w, act));
+}
+__device__ __forceinline__ void store_act4(__nv_bfloat16* y, const float4& v, int act)
+{
+    __nv_bfloat162 h[2] = {__floats2bfloat162_rn(activate(v.x, act), activate(v.y, act)),
+                           __floats2bfloat162_rn(activate(v.z, act), activate(v.w, act))};
+    *reinterpret_cast<uint2*>(y) = *reinterpret_cast<const uint2*>(h);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) warp_pre_kernel(const WarpPreArgs a)
+{
+    constexpr int VX = 16 / (int)sizeof(T);
+    const int LP = 1 << a.lp_log2;
+    const int g = threadIdx.x & (LP - 1);
+    const long long npx = (long long)a.n * a.H * a.W;
+    const long long ngroups = ((long long)gridDim.x * blockDim.x) >> a.lp_log2;
+    // the lanes of a warp iterate together (the change flag is a shuffle reduction over each group)
+    const long long gid = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> a.lp_log2;
+    const long long gid0 = gid - ((threadIdx.x & 31) >> a.lp_log2);
+    const T* xt = static_cast<const T*>(a.xt);
+    const T* xp = static_cast<const T*>(a.xp);
+    T* xn = static_cast<T*>(a.xn);
+    T* y = static_cast<T*>(a.y);
+    for (long long it = 0; gid0 + it < npx; it += ngroups) {
+        const long long p = gid + it;
+        const bool live = p < npx;
+        Bilinear bl = {};
+        if (live) {
+            const int ix = (int)(p % a.W), iy = (int)((p / a.W) % a.H), nn = (int)(p / ((long long)a.W * a.H));
+            bl = bilinear_of(a.flow, nn, a.H, a.W, 1, iy, ix);   // offsets in pixels
         }
-        const bool changed = __any_sync(0xffffffffu, d != 0);
-        if (changed || chg_prev[pix])
-            for (int c = lane; c < C; c += 32) xn[base + c] = xt[base + c];
-        if (lane == 0) chg_cur[pix] = changed ? 1 : 0;
+        if (a.tx) {
+            unsigned d = 0;
+            if (live) {
+                for (int k = g; k < a.C / VX; k += LP) {
+                    const size_t e = (size_t)p * a.C + (size_t)k * VX;
+                    const uint4 av = *reinterpret_cast<const uint4*>(xt + e);
+                    const uint4 bv = *reinterpret_cast<const uint4*>(xp + e);
+                    d |= (av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w);
+                    float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        float f[8];
+                        unpack16(*reinterpret_cast<const uint4*>(xp + bl.off[q] * a.C + (size_t)k * VX), f, (const T*)nullptr);
+#pragma unroll
+                        for (int j = 0; j < VX; ++j) v[j] += bl.wt[q] * f[j];
+                    }
+                    float4* o = reinterpret_cast<float4*>(a.tx + e);
+                    o[0] = make_float4(v[0], v[1], v[2], v[3]);
+                    if (VX == 8) o[1] = make_float4(v[4], v[5], v[6], v[7]);
+                }
+            }
+            for (int o = LP >> 1; o > 0; o >>= 1) d |= __shfl_xor_sync(0xffffffffu, d, o);
+            if (live) {
+                const bool changed = d != 0;
+                if (changed || a.chg_prev[p])
+                    for (int k = g; k < a.C / VX; k += LP) {
+                        const size_t e = (size_t)p * a.C + (size_t)k * VX;
+                        *reinterpret_cast<uint4*>(xn + e) = *reinterpret_cast<const uint4*>(xt + e);
+                    }
+                if (g == 0) a.chg_cur[p] = changed ? 1 : 0;
+            }
+        }
+        if (!live) continue;
+        if ((a.Co & 3) == 0) {
+            for (int k = g; k < a.Co / 4; k += LP) {
+                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 zq = *reinterpret_cast<const float4*>(a.zsrc + bl.off[q] * a.Co + (size_t)k * 4);
+                    v.x += bl.wt[q] * zq.x;
+                    v.y += bl.wt[q] * zq.y;
+                    v.z += bl.wt[q] * zq.z;
+                    v.w += bl.wt[q] * zq.w;
+                }
+                const size_t e = (size_t)p * a.Co + (size_t)k * 4;
+                *reinterpret_cast<float4*>(a.zdst + e) = v;
+                if (y) store_act4(y + e, v, a.act);
+            }
+        } else {
+            for (int c = g; c < a.Co; c += LP) {
+                float v = 0.f;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) v += bl.wt[q] * a.zsrc[bl.off[q] * a.Co + c];
+                const size_t e = (size_t)p * a.Co + c;
+                a.zdst[e] = v;
+                if (y) y[e] = from_f32<T>(activate(v, a.act));
+            }
+        }
     }
 }
 
@@ -1346,8 +1459,8 @@ cudaError_t step_local_prepare(Layer& L)
         if (e == cudaSuccess) e = alloc_ychg(L);
         if (e == cudaSuccess) e = ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
         // warped steps run the staged form's warped variant, or the general form when it does not fit
-        StagedShape tw;
-        if (e == cudaSuccess && staged_ok(L, &tw, true)) e = ensure_dynamic_smem(staged_kernel_of(L, tw.sw, true), tw.smem);
+        StagedShape tp, tw;
+        if (e == cudaSuccess && staged_wp_ok(L, &tp, &tw)) e = ensure_dynamic_smem(staged_kernel_of(L, tw.sw, true), tw.smem);
         if (e == cudaSuccess && choose_shape(L).smem <= LOCAL_MAX_SMEM) e = ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
         return e;
     }
@@ -1357,51 +1470,84 @@ cudaError_t step_local_prepare(Layer& L)
     return ensure_dynamic_smem(kernel_of(L), choose_shape(L).smem);
 }
 
+cudaError_t launch_step_warp_pass(Layer& L, const void* x_t, const void* shortcut, const float* flow)
+{
+    const int cur = (int)(L.t & 1), nxt = cur ^ 1;
+    StagedShape t, tw;
+    const bool staged = staged_wp_ok(L, &t, &tw);
+    const size_t nz = (size_t)L.p.n_streams * L.ho * L.wo * L.p.c_out;
+    const size_t nx = (size_t)L.p.n_streams * L.p.h * L.p.w * L.p.c_in;
+    cudaError_t e = cudaSuccess;
+    if (!L.z_prev) {
+        e = cudaMalloc((void**)&L.z_prev, nz * sizeof(float));
+        if (e != cudaSuccess) {
+            L.z_prev = nullptr;
+            return e;
+        }
+        L.state_bytes += nz * sizeof(float);
+    }
+    if (staged && !L.tx) {
+        e = cudaMalloc((void**)&L.tx, nx * sizeof(float));
+        if (e != cudaSuccess) {
+            L.tx = nullptr;
+            return e;
+        }
+        L.state_bytes += nx * sizeof(float);
+        EncodeTiledFn enc = encode_tiled_fn();
+        const cuuint64_t C = L.p.c_in, W = L.p.w, H = L.p.h, N = L.p.n_streams;
+        cuuint64_t dims[4] = {C, W, H, N};
+        cuuint64_t strides[3] = {C * 4, W * C * 4, H * W * C * 4};
+        cuuint32_t box[4] = {(cuuint32_t)C, (cuuint32_t)tw.g.FW, (cuuint32_t)tw.g.FH, 1};
+        cuuint32_t estr[4] = {1, 1, 1, 1};
+        if (!enc || enc(&L.tmap_tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, L.tx, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+            set_error("tensor map of the warped frame rejected");
+            return cudaErrorInvalidValue;
+        }
+    }
+    WarpPreArgs w;
+    w.flow = flow;
+    w.zsrc = L.z;
+    w.zdst = L.z_prev;
+    w.y = L.y && !shortcut ? L.y : nullptr;
+    w.xt = x_t;
+    w.xp = L.xbuf[cur];
+    w.xn = L.xbuf[nxt];
+    w.chg_prev = L.chg[nxt];
+    w.chg_cur = L.chg[cur];
+    w.tx = staged ? L.tx : nullptr;
+    w.n = L.p.n_streams; w.H = L.p.h; w.W = L.p.w; w.C = L.p.c_in; w.Co = L.p.c_out; w.act = L.p.activation;
+    const int vx = 16 / L.esize;
+    int chunks = (L.p.c_out % 4 == 0) ? L.p.c_out / 4 : L.p.c_out;
+    if (staged) chunks = std::max(chunks, L.p.c_in / vx);
+    w.lp_log2 = 0;
+    while ((1 << w.lp_log2) < chunks && w.lp_log2 < 5) ++w.lp_log2;
+    const long long npx = (long long)L.p.n_streams * L.p.h * L.p.w;
+    const long long per_block = 256 >> w.lp_log2;
+    const long long blocks = (npx + per_block - 1) / per_block, cap = (long long)L.num_sms * 8;
+    const int grid = (int)(blocks < cap ? blocks : cap);
+    if (L.p.dtype == SKIPCONV_BF16) warp_pre_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(w);
+    else warp_pre_kernel<float><<<grid, 256, 0, L.stream>>>(w);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    std::swap(L.z, L.z_prev);
+    if (L.local_staged && !encode_tile_map(&L.tmap_ztile, L.z, L, t, true)) {
+        set_error("tensor map of the layer state rejected");
+        return cudaErrorInvalidValue;
+    }
+    return cudaSuccess;
+}
+
 cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, int force, const Layer* px,
                               const Layer* psc, const float* flow)
 {
     const int cur = (int)(L.t & 1), nxt = cur ^ 1;
     cudaLaunchAttribute attr[1];
     StagedShape t;
-    if (flow && L.local_staged && staged_ok(L, &t, true)) {
-        // warped residual on the staged form: T(x_{t-1}) and the commit first, then the step with the
-        // warped frame as its previous input
-        const size_t nx = (size_t)L.p.n_streams * L.p.h * L.p.w * L.p.c_in;
-        if (!L.tx) {
-            cudaError_t e = cudaMalloc((void**)&L.tx, nx * sizeof(float));
-            if (e != cudaSuccess) {
-                L.tx = nullptr;
-                return e;
-            }
-            L.state_bytes += nx * sizeof(float);
-            EncodeTiledFn enc = encode_tiled_fn();
-            const cuuint64_t C = L.p.c_in, W = L.p.w, H = L.p.h, N = L.p.n_streams;
-            cuuint64_t dims[4] = {C, W, H, N};
-            cuuint64_t strides[3] = {C * 4, W * C * 4, H * W * C * 4};
-            cuuint32_t box[4] = {(cuuint32_t)C, (cuuint32_t)t.g.FW, (cuuint32_t)t.g.FH, 1};
-            cuuint32_t estr[4] = {1, 1, 1, 1};
-            if (!enc || enc(&L.tmap_tx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, L.tx, dims, strides, box, estr,
-                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
-                set_error("tensor map of the warped frame rejected");
-                return cudaErrorInvalidValue;
-            }
-        }
-        const long long npx = (long long)L.p.n_streams * L.p.h * L.p.w;
-        const long long blocks = (npx + 7) / 8, cap = (long long)L.num_sms * 16;
-        const int grid = (int)(blocks < cap ? blocks : cap);
-        if (L.p.dtype == SKIPCONV_BF16)
-            warp_prev_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(
-                (const __nv_bfloat16*)x_t, (const __nv_bfloat16*)L.xbuf[cur], (__nv_bfloat16*)L.xbuf[nxt], L.chg[nxt],
-                L.chg[cur], flow, L.tx, L.p.n_streams, L.p.h, L.p.w, L.p.c_in);
-        else
-            warp_prev_kernel<float><<<grid, 256, 0, L.stream>>>((const float*)x_t, (const float*)L.xbuf[cur],
-                                                                (float*)L.xbuf[nxt], L.chg[nxt], L.chg[cur], flow,
-                                                                L.tx, L.p.n_streams, L.p.h, L.p.w, L.p.c_in);
-        const cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-        return launch_staged(L, t, x_t, shortcut, force, nullptr, nullptr, &L.tmap_tx, true);
-    }
+    StagedShape tw;
+    if (flow && staged_wp_ok(L, &t, &tw))
+        return launch_staged(L, tw, x_t, shortcut, force, nullptr, nullptr, &L.tmap_tx, true);
     if (L.local_staged && !flow) {
         if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
         return launch_staged(L, t, x_t, shortcut, force, px, psc, &L.tmap_fp[cur], false);

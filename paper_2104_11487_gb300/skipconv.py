@@ -118,7 +118,7 @@ def skipconv_profile(handle: int, enable: bool) -> None:
 
 def skipconv_profile_read(handle: int):
     """Returns (launches, ms), lists of PROFILE_KINDS per kernel kind: gate_pixel, gate_block, conv,
-    y_refresh, fused tensor-core step, one-launch CUDA-core step."""
+    y_refresh, fused tensor-core step, one-launch CUDA-core step, warp pass of a warped step."""
     launches = (ctypes.c_longlong * _lib.PROFILE_KINDS)()
     ms = (ctypes.c_double * _lib.PROFILE_KINDS)()
     check("skipconv_profile_read", _lib.lib().skipconv_profile_read(handle, launches, ms))
