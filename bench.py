@@ -547,7 +547,7 @@ def warped_report(torch, flush, steps=12, warmup=3):
 
 
 # ----------------------------------------------------------- CPU oracle
-def cpu_oracle_sample(seconds, density, max_frames=40):
+def cpu_oracle_sample(seconds, density, max_frames=200):
     """The oracle as it stands, on the host cores: stream 0 of the same
     workload, state preset to the frame before the sample (no key frame),
     stepping frames until `seconds` of work or `max_frames`."""
