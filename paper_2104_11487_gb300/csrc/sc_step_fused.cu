@@ -28,10 +28,11 @@
 //
 // Hand-off between CTAs carries its own readiness: a published norm is one
 // 64-bit word (step epoch, fp32 norm) and a gate decision one 32-bit word
-// (step epoch, open bit), each written and read with single-copy-atomic
-// relaxed accesses; a reader polls the words it needs until all carry this
-// step's epoch.  Every step rewrites every word, so no counter, fence or
-// reset is needed, and each hop costs one memory round trip.  Every CTA
+// (step epoch, open bit), each written with a relaxed max reduction at L2 and
+// read with single-copy-atomic relaxed loads; a reader polls the words it needs
+// until all carry this step's epoch.  Every step rewrites every word, so no
+// counter or fence is needed (the words are cleared only before the epoch
+// wraps around), and each hop costs one memory round trip.  Every CTA
 // derives the same ordered list of open blocks from the decisions, so no
 // atomics build it; the CTA that owns stream n (n mod grid) writes that
 // stream's part of the ABI's list.  Every poll is bounded; a CTA that gives
@@ -102,22 +103,20 @@ __device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t* p)
     return v;
 }
 
-// Publish a tagged word for pollers on other SMs.  An atomic exchange is
+// Publish a tagged word for pollers on other SMs: a relaxed max reduction,
 // performed at the word's home in L2, so a poller on either die sees it after
-// one round trip; a plain store was measured to linger for microseconds
-// before other SMs observed it.
+// one round trip (a plain store was measured to linger for microseconds before
+// other SMs observed it).  The step epoch sits in the high bits and only grows
+// between resets of the words, so the maximum is the new word.  A reduction
+// returns nothing: the writing warp does not wait for the round trip.
 __device__ __forceinline__ void publish_u64(uint64_t* p, uint64_t v)
 {
-    uint64_t o;
-    asm volatile("atom.relaxed.gpu.global.exch.b64 %0, [%1], %2;" : "=l"(o) : "l"(p), "l"(v) : "memory");
-    (void)o;
+    asm volatile("red.relaxed.gpu.global.max.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
 __device__ __forceinline__ void publish_u32(uint32_t* p, uint32_t v)
 {
-    uint32_t o;
-    asm volatile("atom.relaxed.gpu.global.exch.b32 %0, [%1], %2;" : "=r"(o) : "l"(p), "r"(v) : "memory");
-    (void)o;
+    asm volatile("red.relaxed.gpu.global.max.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ uint4 ld_relaxed_v4(const uint32_t* p)
@@ -618,7 +617,15 @@ cudaError_t launch_step_fused(Layer& L, const void* x_t, int force)
         set_error("tensor map of x_t rejected");
         return cudaErrorInvalidValue;
     }
-    L.epoch = L.epoch % 0x7fffffffu + 1u;   // 1 .. 2^31 - 1; every step rewrites every tagged word
+    // 1 .. 2^31 - 1; every step rewrites every tagged word with a max reduction, so the words go back
+    // to 0 (no epoch) before the epoch wraps around to 1
+    if (L.epoch == 0x7fffffffu) {
+        cudaError_t e = cudaMemsetAsync(L.pnorm, 0, (size_t)L.p.n_streams * L.p.h * L.p.w * sizeof(uint64_t), L.stream);
+        if (e == cudaSuccess)
+            e = cudaMemsetAsync(L.gtag, 0, (size_t)L.p.n_streams * L.nby * L.nbx * sizeof(uint32_t), L.stream);
+        if (e != cudaSuccess) return e;
+    }
+    L.epoch = L.epoch % 0x7fffffffu + 1u;
     const int cur = (int)(L.t & 1), nxt = cur ^ 1;
     FusedArgs a;
     a.xt = (const uint8_t*)x_t;

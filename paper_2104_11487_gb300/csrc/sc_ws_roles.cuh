@@ -329,7 +329,9 @@ __device__ __forceinline__ void epilogue_role(float* sZ, Bars* b, uint32_t tmem,
             ptx::bulk_commit_group();
         }
     }
-    if (tid == 0) ptx::bulk_wait_group0();
+    // the staging tile must stay valid until the last reduce-add has read it; its writes to z~ complete
+    // with the grid
+    if (tid == 0) ptx::bulk_wait_group_read0();
 }
 
 }  // namespace ws
