@@ -789,6 +789,13 @@ def main():
     # 6) the CPU oracle on the host cores (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_oracle_sample(args.cpu_seconds, args.density)
+        # the same oracle on one host core (a shorter sample)
+        import oracle
+        cores = oracle.num_threads()
+        oracle.set_num_threads(1)
+        one = cpu_oracle_sample(args.cpu_seconds / 3, args.density)
+        oracle.set_num_threads(cores)
+        line["cpu_baseline"]["single_core"] = {"value": one["value"], "unit": one["unit"], "sample": one["sample"]}
     layer.close()
     if args.drift and rank == 0:
         line["drift_vs_dense"] = drift_report(torch)
