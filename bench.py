@@ -70,6 +70,8 @@ def parse():
     ap.add_argument("--no-soak", action="store_true",
                     help="skip the untimed steps around the timed region (for profiler runs)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--clocks-log", default=None, metavar="PATH",
+                    help="keep the nvidia-smi samples of the timed region in this CSV (default: a temporary file)")
     return ap.parse_args()
 
 
@@ -101,13 +103,17 @@ class Clocks:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index):
-        self.index, self.proc, self.path = index, None, None
+    def __init__(self, index, path=None):
+        self.index, self.proc, self.path = index, None, path
 
     def start(self):
         try:
-            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-            self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_%d.csv" % os.getpid())
+            if self.path is None:
+                import tempfile
+                fd, self.path = tempfile.mkstemp(prefix="clocks_bench_", suffix=".csv")
+                os.close(fd)
+            else:
+                os.makedirs(os.path.dirname(os.path.abspath(self.path)), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
                                           "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
@@ -664,7 +670,7 @@ def main():
     info = skipconv_get_info(layer.handle)
 
     # 1) headline: timed steps, no per-kernel events
-    clocks = Clocks(local)
+    clocks = Clocks(local, args.clocks_log)
     barrier()
     clocks.start()
     if not args.no_soak:
