@@ -44,8 +44,9 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--density", type=float, default=0.10)
-    ap.add_argument("--gate", choices=("input", "output"), default="input",
-                    help="input: Input-Norm gate (Eq. 5, mean over the support); output: Output-Norm gate (Eq. 7)")
+    ap.add_argument("--gate", choices=("input", "output", "gumbel"), default="input",
+                    help="input: Input-Norm gate (Eq. 5, mean over the support); output: Output-Norm gate (Eq. 7); "
+                         "gumbel: the Gumbel gate at inference (Eq. 8) with a seeded random phi (separate launches)")
     ap.add_argument("--key-interval", type=int, default=0,
                     help="a key frame every K steps (Table 4's periodic reset); 0: none after the first")
     ap.add_argument("--drift", action="store_true",
@@ -79,7 +80,8 @@ def workload_config(density, flushed=True, gate="input", key_interval=0):
     return {"workload": "c4: 3x3 Skip-Conv 256->256, %d streams x %dx%d, bf16 (fp32 accum), %dx%d blocks, "
                         "eps %.2g, %g%% block density" % (N_STREAMS, H, W, BLOCK, BLOCK, EPS, density * 100),
             "streams": N_STREAMS, "h": H, "w": W, "c_in": C, "c_out": C, "k": K, "block": BLOCK, "eps": EPS,
-            "gate": {"input": "input-norm (mean over support)", "output": "output-norm (Eq. 7)"}[gate],
+            "gate": {"input": "input-norm (mean over support)", "output": "output-norm (Eq. 7)",
+                     "gumbel": "gumbel at inference (Eq. 8), f(r; phi) > eps, phi ~ N(0, 1/(9 c_in)) seeded, bias 0"}[gate],
             "key_interval": key_interval, "density": density,
             "l2": ("flushed between timed steps (256 MiB written, then read back)" if flushed else
                    "not flushed: each step streams two 64 MiB frames per step in stream order, more than the 129 MB L2"),
@@ -235,14 +237,20 @@ LAUNCH_FORMS = {0: "separate gate and convolution launches", 1: "one cooperative
                 2: "one CUDA-core launch (a CTA per tile of gate blocks)"}
 
 
-GATES = {"input": 0, "output": 2}         # Input-Norm (mean), Output-Norm
+GATES = {"input": 0, "output": 2, "gumbel": 3}   # Input-Norm (mean), Output-Norm, Gumbel (Eq. 8)
 
 
 def make_layer(wl, torch, dense_mode=False, path="fused", gate="input", key_interval=0):
     from paper_2104_11487_gb300 import SkipConvLayer
+    phi = None
+    if gate == "gumbel":
+        # the gate function of Eq. 8 has no trained weights here: a seeded random one-output-channel conv
+        rng = np.random.default_rng(7001)
+        phi = torch.from_numpy((rng.standard_normal((1, C, K, K)) / np.sqrt(K * K * C)).astype(np.float32))
     return SkipConvLayer(N_STREAMS, C, C, H, W, k=K, stride=1, pad=1, block=BLOCK, eps=EPS, dtype="bf16",
                          dense_mode=dense_mode, conv_path=CONV_PATH[path], gate=GATES[gate],
-                         key_interval=key_interval, weights=torch.from_numpy(wl.weights[0]), bias=None)
+                         key_interval=key_interval, weights=torch.from_numpy(wl.weights[0]), bias=None,
+                         gate_weights=phi, gate_bias=0.0)
 
 
 PROFILE_FILES = {"gate_pixel": ("gate_pixel", ("sc_gate.cu",)), "gate_block": ("gate_block", ("sc_gate.cu",)),
@@ -719,9 +727,12 @@ def main():
                 "traffic": traffic_from_profiles("conv")}
     else:
         ach = gate_bytes / (dom_us * 1e-6) / 1e9 if dom == 0 else None
-        roof = {"kernel": KERNELS[dom], "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+        # the Gumbel gate's passes are other kernels than the ones the committed summaries profile
+        name = KERNELS[dom] + ("_gumbel" if args.gate == "gumbel" else "")
+        roof = {"kernel": name, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                 "frac": (ach / hbm) if ach else None, "peak_source": pk_src + " hbm_gbs",
-                "algorithmic_bytes_per_launch": gate_bytes, "traffic": traffic_from_profiles(KERNELS[dom])}
+                "algorithmic_bytes_per_launch": gate_bytes,
+                "traffic": None if args.gate == "gumbel" else traffic_from_profiles(KERNELS[dom])}
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",

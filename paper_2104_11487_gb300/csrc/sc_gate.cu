@@ -340,6 +340,153 @@ __global__ void __launch_bounds__(256) gate_pixel_gumbel_kernel(
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// The same pass for pixels of 16-byte vectors: G = 2^LOG2G lanes per pixel
+// (8 to 32), each with one 16-byte vector of both frames, 32 / G pixels per
+// warp.  A lane forms its channels' share of all taps (phi from shared
+// memory, four floats per load); the pixel's G shares of taps 0-7 are summed
+// by a transposed butterfly (three halving exchanges leave one tap's partial
+// sum in each lane, then plain steps) and tap 8 by a plain one, so every tap
+// costs a fraction of a butterfly of its own.
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8], const __nv_bfloat16*)
+{
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 t = __bfloat1622float2(h[k]);
+        f[2 * k] = t.x;
+        f[2 * k + 1] = t.y;
+    }
+}
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8], const float*)
+{
+    f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y); f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+    f[4] = f[5] = f[6] = f[7] = 0.f;
+}
+
+template <typename T, int LOG2G>
+__global__ void __launch_bounds__(256) gate_pixel_gumbel_vec_kernel(
+    const T* __restrict__ xt, const T* __restrict__ xp, T* __restrict__ xn, const uint8_t* __restrict__ chg_prev,
+    uint8_t* __restrict__ chg_cur, const float* __restrict__ phi, float* __restrict__ taps_out, long long n_pix, int C,
+    int taps, int32_t* __restrict__ count_cur, int32_t* __restrict__ count_next)
+{
+    constexpr int G = 1 << LOG2G, PPW = 32 / G, VX = 16 / (int)sizeof(T);
+    constexpr int PL = 2;   // pixels per lane and pass: their loads go out together, phi is read once for both
+    extern __shared__ float sphi[];  // [GUMBEL_MAX_TAPS][C], taps past `taps` zero
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        *count_cur = 0;
+        *count_next = 0;
+    }
+    for (int i = threadIdx.x; i < GUMBEL_MAX_TAPS * C; i += blockDim.x) sphi[i] = i < taps * C ? phi[i] : 0.f;
+    __syncthreads();
+    const int lane = threadIdx.x & 31, sub = lane & (G - 1), prow = lane >> LOG2G;
+    const int units = C / VX;
+    const bool lane_on = sub < units;
+    const int c0 = sub * VX;
+    // the tap whose sum this lane holds after the halving exchanges
+    const int my_tap = (((sub >> (LOG2G - 1)) & 1) << 2) | (((sub >> (LOG2G - 2)) & 1) << 1) | ((sub >> (LOG2G - 3)) & 1);
+    const bool writer = (sub & ((G >> 3) - 1)) == 0;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    for (long long p0 = warp * PPW * PL; p0 < n_pix; p0 += nwarps * PPW * PL) {
+        long long pix[PL];
+        bool on[PL];
+        uint4 av[PL], bv[PL];
+#pragma unroll
+        for (int u = 0; u < PL; ++u) {
+            pix[u] = p0 + u * PPW + prow;
+            on[u] = lane_on && pix[u] < n_pix;
+            av[u] = make_uint4(0, 0, 0, 0);
+            bv[u] = av[u];
+            if (on[u]) {
+                av[u] = reinterpret_cast<const uint4*>(xt + pix[u] * C)[sub];
+                bv[u] = reinterpret_cast<const uint4*>(xp + pix[u] * C)[sub];
+            }
+        }
+        float r[PL][8], acc[PL][GUMBEL_MAX_TAPS];
+        unsigned d[PL];
+#pragma unroll
+        for (int u = 0; u < PL; ++u) {
+            d[u] = (av[u].x ^ bv[u].x) | (av[u].y ^ bv[u].y) | (av[u].z ^ bv[u].z) | (av[u].w ^ bv[u].w);
+            float fa[8], fb[8];
+            unpack8(av[u], fa, (const T*)nullptr);
+            unpack8(bv[u], fb, (const T*)nullptr);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) r[u][j] = fa[j] - fb[j];
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) acc[u][t] = 0.f;
+        }
+        if (lane_on) {
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) {
+                const float4 w0 = *reinterpret_cast<const float4*>(sphi + t * C + c0);
+                const float4 w1 = VX == 8 ? *reinterpret_cast<const float4*>(sphi + t * C + c0 + 4)
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int u = 0; u < PL; ++u) {
+                    float a = 0.f;
+                    a = fmaf(w0.x, r[u][0], a);
+                    a = fmaf(w0.y, r[u][1], a);
+                    a = fmaf(w0.z, r[u][2], a);
+                    a = fmaf(w0.w, r[u][3], a);
+                    if (VX == 8) {
+                        a = fmaf(w1.x, r[u][4], a);
+                        a = fmaf(w1.y, r[u][5], a);
+                        a = fmaf(w1.z, r[u][6], a);
+                        a = fmaf(w1.w, r[u][7], a);
+                    }
+                    acc[u][t] = a;
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < PL; ++u) {
+            // taps 0-7: transposed butterfly over the pixel's G lanes
+            float t4[4], t2[2], t1;
+            {
+                const bool h = (sub >> (LOG2G - 1)) & 1;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float send = h ? acc[u][q] : acc[u][q + 4], keep = h ? acc[u][q + 4] : acc[u][q];
+                    t4[q] = keep + __shfl_xor_sync(0xffffffffu, send, G >> 1);
+                }
+            }
+            {
+                const bool h = (sub >> (LOG2G - 2)) & 1;
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                    const float send = h ? t4[q] : t4[q + 2], keep = h ? t4[q + 2] : t4[q];
+                    t2[q] = keep + __shfl_xor_sync(0xffffffffu, send, G >> 2);
+                }
+            }
+            {
+                const bool h = (sub >> (LOG2G - 3)) & 1;
+                const float send = h ? t2[0] : t2[1], keep = h ? t2[1] : t2[0];
+                t1 = keep + __shfl_xor_sync(0xffffffffu, send, G >> 3);
+            }
+#pragma unroll
+            for (int off = G >> 4; off > 0; off >>= 1) t1 += __shfl_xor_sync(0xffffffffu, t1, off);
+            // tap 8 and the change bits: plain butterflies within the pixel's lanes
+            float a8 = acc[u][8];
+            unsigned du = d[u];
+#pragma unroll
+            for (int off = G >> 1; off > 0; off >>= 1) {
+                a8 += __shfl_xor_sync(0xffffffffu, a8, off);
+                du |= __shfl_xor_sync(0xffffffffu, du, off);
+            }
+            if (pix[u] < n_pix) {
+                const bool changed = du != 0;
+                if (on[u] && (changed || chg_prev[pix[u]])) reinterpret_cast<uint4*>(xn + pix[u] * C)[sub] = av[u];
+                if (writer && my_tap < taps) taps_out[pix[u] * taps + my_tap] = t1;
+                if (sub == 0) {
+                    if (taps > 8) taps_out[pix[u] * taps + 8] = a8;
+                    chg_cur[pix[u]] = changed ? 1 : 0;
+                }
+            }
+        }
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Gumbel gate, pass 2 of 2: one warp per gate block.  f at an output location
 // is phi_bias plus the partial products of the taps over its receptive field
 // (zero padding: out-of-frame taps add nothing); the block opens when its
@@ -503,7 +650,21 @@ int gate_max_channels(int dtype, bool vec)
     return vec ? (32 * 4 * 16) / es : 32 * 32;
 }
 
-size_t gumbel_smem_bytes(const Layer& L) { return (size_t)L.p.k_h * L.p.k_w * L.p.c_in * sizeof(float); }
+size_t gumbel_smem_bytes(const Layer& L)
+{
+    return (size_t)(L.p.k_h * L.p.k_w > GUMBEL_MAX_TAPS ? L.p.k_h * L.p.k_w : GUMBEL_MAX_TAPS) * L.p.c_in * sizeof(float);
+}
+
+// lanes per pixel of the vector form (2^k, 8 to 32), or 0 when the pixel is not whole 16-byte vectors
+static int gumbel_vec_log2g(const Layer& L)
+{
+    if ((L.p.c_in * L.esize) % 16 != 0) return 0;
+    const int units = L.p.c_in * L.esize / 16;
+    if (units > 32) return 0;
+    int lg = 3;
+    while ((1 << lg) < units) ++lg;
+    return lg;
+}
 
 cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
                                       const uint8_t* chg_prev, uint8_t* chg_cur)
@@ -514,6 +675,27 @@ cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const voi
     const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
     const size_t smem = gumbel_smem_bytes(L);
     const int taps = L.p.k_h * L.p.k_w;
+    const int lg = taps <= GUMBEL_MAX_TAPS ? gumbel_vec_log2g(L) : 0;
+    if (lg) {
+        const long long per_block = 16LL * (32 >> lg);   // pixels per CTA pass (two per lane group)
+        const long long vblocks = (n_pix + per_block - 1) / per_block;
+        const int vgrid = (int)(vblocks < cap ? (vblocks > 0 ? vblocks : 1) : cap);
+#define SC_GUMBEL_VEC(T, LG)                                                                                       \
+    gate_pixel_gumbel_vec_kernel<T, LG><<<vgrid, 256, smem, L.stream>>>(                                            \
+        (const T*)x_t, (const T*)x_prev, (T*)x_next, chg_prev, chg_cur, L.gphi, L.pix_taps, n_pix, L.p.c_in, taps,   \
+        step_count(L), next_count(L))
+        if (L.p.dtype == SKIPCONV_BF16) {
+            if (lg == 5) SC_GUMBEL_VEC(__nv_bfloat16, 5);
+            else if (lg == 4) SC_GUMBEL_VEC(__nv_bfloat16, 4);
+            else SC_GUMBEL_VEC(__nv_bfloat16, 3);
+        } else {
+            if (lg == 5) SC_GUMBEL_VEC(float, 5);
+            else if (lg == 4) SC_GUMBEL_VEC(float, 4);
+            else SC_GUMBEL_VEC(float, 3);
+        }
+#undef SC_GUMBEL_VEC
+        return cudaGetLastError();
+    }
     if (L.p.dtype == SKIPCONV_BF16)
         gate_pixel_gumbel_kernel<__nv_bfloat16><<<grid, 256, smem, L.stream>>>(
             (const __nv_bfloat16*)x_t, (const __nv_bfloat16*)x_prev, (__nv_bfloat16*)x_next, chg_prev, chg_cur,

@@ -175,6 +175,9 @@ GUMBEL_CASES = [
     ("bf16_b8", 1, 48, 40, 64, 64, 1, 8, "bf16"),
     ("f32_b1", 1, 32, 24, 32, 32, 1, 1, "f32"),
     ("f32_stride2_ragged", 2, 37, 29, 16, 24, 2, 4, "f32"),
+    # 32 lanes per pixel in the vector form; and a pixel that is not whole 16-byte vectors (scalar form)
+    ("bf16_c256_b8", 1, 24, 32, 256, 32, 1, 8, "bf16"),
+    ("bf16_c12_b2", 1, 20, 18, 12, 16, 1, 2, "bf16"),
 ]
 
 
