@@ -183,6 +183,24 @@ SKIPCONV_API int skipconv_link_inputs(skipconv_handle h, skipconv_handle produce
  * returning.  The first call allocates a device staging frame. */
 SKIPCONV_API int skipconv_step_host(skipconv_handle h, const void* x_t_host, float* z_out_host);
 
+/* Pipelined host-buffer step: the same work as skipconv_step_host, enqueued
+ * without waiting.  The copy of x_t_host (host, [n][h][w][c_in] dtype;
+ * pinned memory, else the copy is synchronous) goes to one of two device
+ * staging frames on the handle's upload stream; the step runs on the
+ * handle's stream once that copy is done; z is then copied on the device to
+ * one of two staging buffers and from there to z_out_host (host float32
+ * [n][ho][wo][c_out], pinned; may be NULL) on the download stream.  So the
+ * upload of step t+1 and the download of step t-1 overlap step t.  Both host
+ * buffers are lent until skipconv_sync returns.  The first call allocates
+ * the staging buffers (2 frames of x, 2 of z) and the two copy streams.
+ * Errors: INVALID (NULL handle or x_t_host), OOM, CUDA; a device error word
+ * set by an earlier step is reported as by skipconv_step. */
+SKIPCONV_API int skipconv_step_host_async(skipconv_handle h, const void* x_t_host, float* z_out_host);
+
+/* Wait for every step and copy enqueued on the handle's streams; reports the
+ * device error word (SKIPCONV_OK, SKIPCONV_ERR_TIMEOUT, SKIPCONV_ERR_DEVICE). */
+SKIPCONV_API int skipconv_sync(skipconv_handle h);
+
 /* The Gumbel gate's function (Eq. 8): phi_oihw, device float32
  * [1][c_in][k_h][k_w] (one output channel, the layer's kernel size), and its
  * bias.  Required before the first step of a SKIPCONV_GATE_GUMBEL layer; may

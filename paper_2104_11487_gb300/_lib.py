@@ -28,6 +28,8 @@ SIGNATURES = {
     "skipconv_reset_state": (c_int, [c_void_p]),
     "skipconv_step": (c_int, [c_void_p, c_void_p, c_void_p]),
     "skipconv_step_host": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "skipconv_step_host_async": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "skipconv_sync": (c_int, [c_void_p]),
     "skipconv_destroy": (c_int, [c_void_p]),
     "skipconv_get_z": (c_int, [c_void_p, c_void_p]),
     "skipconv_get_y": (c_int, [c_void_p, c_void_p]),

@@ -633,6 +633,98 @@ int skipconv_step_host(skipconv_handle h, const void* x_t_host, float* z_out_hos
     return check_device_word(L);
 }
 
+static void async_release(Layer* L);
+
+// Copy streams, events and staging buffers of the pipelined host step (first call).
+static cudaError_t async_prepare(Layer* L)
+{
+    if (L->up_stream) return cudaSuccess;
+    const size_t xbytes = (size_t)L->p.n_streams * L->p.h * L->p.w * L->p.c_in * L->esize;
+    const size_t zbytes = (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * sizeof(float);
+    cudaError_t e = cudaSuccess;
+    for (int s = 0; s < 2 && e == cudaSuccess; ++s) {
+        e = cudaMalloc(&L->xs_async[s], xbytes);
+        if (e != cudaSuccess) L->xs_async[s] = nullptr;
+        if (e == cudaSuccess) {
+            e = cudaMalloc((void**)&L->zs_async[s], zbytes);
+            if (e != cudaSuccess) L->zs_async[s] = nullptr;
+        }
+        for (cudaEvent_t* ev : {&L->ev_up[s], &L->ev_used[s], &L->ev_zready[s], &L->ev_down[s]})
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+    }
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&L->down_stream, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&L->up_stream, cudaStreamNonBlocking);
+    if (e == cudaSuccess) L->state_bytes += 2 * (xbytes + zbytes);
+    else async_release(L);
+    return e;
+}
+
+static void async_release(Layer* L)
+{
+    for (cudaStream_t st : {L->up_stream, L->down_stream})
+        if (st) {
+            cudaStreamSynchronize(st);
+            cudaStreamDestroy(st);
+        }
+    L->up_stream = L->down_stream = nullptr;
+    for (int s = 0; s < 2; ++s) {
+        for (cudaEvent_t ev : {L->ev_up[s], L->ev_used[s], L->ev_zready[s], L->ev_down[s]})
+            if (ev) cudaEventDestroy(ev);
+        L->ev_up[s] = L->ev_used[s] = L->ev_zready[s] = L->ev_down[s] = nullptr;
+        if (L->xs_async[s]) cudaFree(L->xs_async[s]);
+        if (L->zs_async[s]) cudaFree(L->zs_async[s]);
+        L->xs_async[s] = nullptr;
+        L->zs_async[s] = nullptr;
+    }
+}
+
+int skipconv_step_host_async(skipconv_handle h, const void* x_t_host, float* z_out_host)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!x_t_host) return set_error("x_t_host is NULL"), SKIPCONV_ERR_INVALID;
+    cudaError_t e = async_prepare(L);
+    if (e != cudaSuccess) return status_of(e);
+    const size_t xbytes = (size_t)L->p.n_streams * L->p.h * L->p.w * L->p.c_in * L->esize;
+    const size_t zbytes = (size_t)L->p.n_streams * L->ho * L->wo * L->p.c_out * sizeof(float);
+    const int s = (int)(L->async_steps & 1);
+    // upload into staging frame s once the step two calls back has read it (an event never recorded
+    // is complete, so the first two calls do not wait)
+    e = cudaStreamWaitEvent(L->up_stream, L->ev_used[s], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(L->xs_async[s], x_t_host, xbytes, cudaMemcpyHostToDevice, L->up_stream);
+    if (e == cudaSuccess) e = cudaEventRecord(L->ev_up[s], L->up_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(L->stream, L->ev_up[s], 0);
+    if (e != cudaSuccess) return status_of(e);
+    int st = skipconv_step(h, L->xs_async[s], nullptr);
+    if (st) return st;
+    e = cudaEventRecord(L->ev_used[s], L->stream);
+    if (e == cudaSuccess && z_out_host) {
+        // z after this step into staging buffer s (free once the download two calls back is done),
+        // then to the host on the download stream
+        e = cudaStreamWaitEvent(L->stream, L->ev_down[s], 0);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(L->zs_async[s], L->z, zbytes, cudaMemcpyDeviceToDevice, L->stream);
+        if (e == cudaSuccess) e = cudaEventRecord(L->ev_zready[s], L->stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(L->down_stream, L->ev_zready[s], 0);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(z_out_host, L->zs_async[s], zbytes, cudaMemcpyDeviceToHost, L->down_stream);
+        if (e == cudaSuccess) e = cudaEventRecord(L->ev_down[s], L->down_stream);
+    }
+    if (e != cudaSuccess) return status_of(e);
+    L->async_steps += 1;
+    return SKIPCONV_OK;
+}
+
+int skipconv_sync(skipconv_handle h)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    cudaError_t e = cudaSuccess;
+    for (cudaStream_t st : {L->up_stream, L->stream, L->down_stream})
+        if (st && e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (!L->up_stream && e == cudaSuccess) e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    return check_device_word(L);
+}
+
 int skipconv_destroy(skipconv_handle h)
 {
     if (!h) return SKIPCONV_OK;
@@ -652,6 +744,7 @@ int skipconv_destroy(skipconv_handle h)
     }
     cudaError_t e = cudaStreamSynchronize(L->stream);
     int st = e == cudaSuccess ? check_device_word(L) : status_of(e);
+    async_release(L);
     free_buffers(L);
     delete h;
     return st;

@@ -43,6 +43,13 @@ struct Layer {
     __nv_bfloat16* w_tc;    // [co_pad][k_h*k_w*ci_pad] bf16 (tensor-core path)
     int ci_pad, co_pad;     // tensor-core padding of c_in (multiple of 64) and c_out (of 128)
     void* x_stage;          // device staging frame for skipconv_step_host (lazy)
+    // skipconv_step_host_async (lazy): staging frames of x and z, copy streams, and per slot the events
+    // "x uploaded", "x consumed by the step", "z staged", "z downloaded"
+    void* xs_async[2];
+    float* zs_async[2];
+    cudaStream_t up_stream, down_stream;
+    cudaEvent_t ev_up[2], ev_used[2], ev_zready[2], ev_down[2];
+    long long async_steps;
     size_t state_bytes;
 
     // error word: pinned, mapped host memory

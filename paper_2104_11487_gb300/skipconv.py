@@ -46,6 +46,15 @@ def skipconv_step_host(handle: int, x_t_host, z_out_host=None) -> None:
     check("skipconv_step_host", _lib.lib().skipconv_step_host(handle, _ptr(x_t_host), _ptr(z_out_host)))
 
 
+def skipconv_step_host_async(handle: int, x_t_host, z_out_host=None) -> None:
+    check("skipconv_step_host_async",
+          _lib.lib().skipconv_step_host_async(handle, _ptr(x_t_host), _ptr(z_out_host)))
+
+
+def skipconv_sync(handle: int) -> None:
+    check("skipconv_sync", _lib.lib().skipconv_sync(handle))
+
+
 def skipconv_destroy(handle: int) -> int:
     return _lib.lib().skipconv_destroy(handle)
 
