@@ -650,20 +650,22 @@ int gate_max_channels(int dtype, bool vec)
     return vec ? (32 * 4 * 16) / es : 32 * 32;
 }
 
-size_t gumbel_smem_bytes(const Layer& L)
-{
-    return (size_t)(L.p.k_h * L.p.k_w > GUMBEL_MAX_TAPS ? L.p.k_h * L.p.k_w : GUMBEL_MAX_TAPS) * L.p.c_in * sizeof(float);
-}
-
 // lanes per pixel of the vector form (2^k, 8 to 32), or 0 when the pixel is not whole 16-byte vectors
 static int gumbel_vec_log2g(const Layer& L)
 {
-    if ((L.p.c_in * L.esize) % 16 != 0) return 0;
+    if ((L.p.c_in * L.esize) % 16 != 0 || L.p.k_h * L.p.k_w > GUMBEL_MAX_TAPS) return 0;
     const int units = L.p.c_in * L.esize / 16;
     if (units > 32) return 0;
     int lg = 3;
     while ((1 << lg) < units) ++lg;
     return lg;
+}
+
+// phi in shared memory: [taps][c_in]; the vector form pads it to GUMBEL_MAX_TAPS taps (c_in <= 256 there)
+size_t gumbel_smem_bytes(const Layer& L)
+{
+    const int taps = gumbel_vec_log2g(L) ? GUMBEL_MAX_TAPS : L.p.k_h * L.p.k_w;
+    return (size_t)taps * L.p.c_in * sizeof(float);
 }
 
 cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
@@ -675,7 +677,7 @@ cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const voi
     const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
     const size_t smem = gumbel_smem_bytes(L);
     const int taps = L.p.k_h * L.p.k_w;
-    const int lg = taps <= GUMBEL_MAX_TAPS ? gumbel_vec_log2g(L) : 0;
+    const int lg = gumbel_vec_log2g(L);
     if (lg) {
         const long long per_block = 16LL * (32 >> lg);   // pixels per CTA pass (two per lane group)
         const long long vblocks = (n_pix + per_block - 1) / per_block;
