@@ -248,6 +248,17 @@ SKIPCONV_API int skipconv_get_stats(skipconv_handle h, long long* active_blocks,
  * SKIPCONV_OK, SKIPCONV_ERR_TIMEOUT or SKIPCONV_ERR_DEVICE. */
 SKIPCONV_API int skipconv_check_device(skipconv_handle h);
 
+/* Failure-detection self-test: launches, on the handle's stream, one kernel
+ * whose bounded wait (the shared-memory barrier wait every pipelined kernel
+ * of the library uses) is never satisfied.  It gives up after limit_ns
+ * (1 .. 1e9) and records a timeout in the handle's device error word, as a
+ * stuck step would; no memory is touched but that word.  Synchronises and
+ * returns what skipconv_check_device then reports: SKIPCONV_ERR_TIMEOUT.
+ * From then on the handle refuses work (steps and resets return the same
+ * status) and is only fit for skipconv_destroy; the CUDA context and other
+ * handles stay usable.  Errors: INVALID (NULL handle, limit out of range). */
+SKIPCONV_API int skipconv_selftest_timeout(skipconv_handle h, long long limit_ns);
+
 /* Per-kernel timing.  Kernel kinds: 0 gate_pixel (residual, channel l1 norm,
  * state commit), 1 gate_block (support norm, block gate, compaction), 2 the
  * convolution of the open blocks (either path), 3 y refresh, 4 the fused

@@ -6,7 +6,7 @@ import os
 
 from . import _build
 
-c_int, c_void_p, c_float = ctypes.c_int, ctypes.c_void_p, ctypes.c_float
+c_int, c_void_p, c_float, c_longlong = ctypes.c_int, ctypes.c_void_p, ctypes.c_float, ctypes.c_longlong
 
 SKIPCONV_OK = 0
 SKIPCONV_ERR_INVALID = -1
@@ -38,6 +38,7 @@ SIGNATURES = {
     "skipconv_get_info": (c_int, [c_void_p, c_void_p]),
     "skipconv_get_stats": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
     "skipconv_check_device": (c_int, [c_void_p]),
+    "skipconv_selftest_timeout": (c_int, [c_void_p, c_longlong]),
     "skipconv_profile": (c_int, [c_void_p, c_int]),
     "skipconv_profile_read": (c_int, [c_void_p, c_void_p, c_void_p]),
     "skipconv_gate_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),

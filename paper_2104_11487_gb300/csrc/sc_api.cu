@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "sc_internal.h"
+#include "sc_ptx.cuh"
 
 namespace sc {
 
@@ -869,6 +870,37 @@ int skipconv_check_device(skipconv_handle h)
     Layer* L = get(h);
     if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
     cudaError_t e = cudaStreamSynchronize(L->stream);
+    if (e != cudaSuccess) return status_of(e);
+    return check_device_word(L);
+}
+
+namespace sc {
+namespace {
+// One bounded wait on a barrier that nothing completes: it runs out after limit_ns and records the timeout in
+// the error word, the path every stuck wait of the library's kernels takes.
+__global__ void selftest_wait_kernel(int* err, unsigned long long limit_ns)
+{
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(ptx::smem_u32(&bar), 1);
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) ptx::mbar_wait(ptx::smem_u32(&bar), 0, nullptr, err, limit_ns);
+}
+}  // namespace
+}  // namespace sc
+
+int skipconv_selftest_timeout(skipconv_handle h, long long limit_ns)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (limit_ns < 1 || limit_ns > 1000000000LL)
+        return set_error("limit_ns must be in 1 .. 1e9"), SKIPCONV_ERR_INVALID;
+    if (int st = check_device_word(L)) return st;
+    selftest_wait_kernel<<<1, 32, 0, L->stream>>>(L->err_dev, (unsigned long long)limit_ns);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaStreamSynchronize(L->stream);
     if (e != cudaSuccess) return status_of(e);
     return check_device_word(L);
 }

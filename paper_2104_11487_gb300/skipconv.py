@@ -121,6 +121,11 @@ def skipconv_check_device(handle: int) -> int:
     return _lib.lib().skipconv_check_device(handle)
 
 
+def skipconv_selftest_timeout(handle: int, limit_ns: int) -> int:
+    """Status of a kernel whose bounded wait runs out (SKIPCONV_ERR_TIMEOUT); the handle is then spent."""
+    return _lib.lib().skipconv_selftest_timeout(handle, int(limit_ns))
+
+
 def skipconv_profile(handle: int, enable: bool) -> None:
     check("skipconv_profile", _lib.lib().skipconv_profile(handle, int(bool(enable))))
 
