@@ -303,6 +303,7 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         const size_t taps = (size_t)L.p.k_h * L.p.k_w;
         e = A.dev((void**)&L.pix_taps, npix * taps * sizeof(float));
         if (e == cudaSuccess) e = A.dev((void**)&L.gphi, taps * L.p.c_in * sizeof(float));
+        if (e == cudaSuccess) e = gumbel_prepare(L);
     }
     if (e == cudaSuccess) e = A.dev((void**)&L.mask, nblk);
     if (e == cudaSuccess) e = A.dev((void**)&L.list, nblk * sizeof(int32_t));

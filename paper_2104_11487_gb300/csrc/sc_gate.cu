@@ -20,6 +20,7 @@
 // publication (fence, atomic, barrier) as on the streaming itself at these
 // frame sizes, and were twice as slow.
 #include "sc_internal.h"
+#include "sc_ptx.cuh"
 
 namespace sc {
 namespace {
@@ -487,6 +488,189 @@ __global__ void __launch_bounds__(256) gate_pixel_gumbel_vec_kernel(
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// The same pass for 512-byte pixels (32 lanes x 16 bytes: 256 bf16 or 128
+// fp32 channels), streamed: a persistent grid of one CTA per SM, each warp
+// refilling its own GS_NSLOT shared-memory slots by bulk copies with chunks of
+// GS_ROWS pixels of both frames, so the bytes in flight do not occupy registers.  A
+// warp takes a whole chunk at once: phi is read once per chunk and shared by
+// its GS_ROWS pixels, and the GS_ROWS x 9 tap sums are reduced over the 32
+// lanes by a transposed butterfly (halving exchanges leave one pixel's 9 sums in
+// each lane, then plain steps).  Waits are bounded; one that runs out
+// records a timeout in the error word.
+constexpr int GS_WARPS = 8;
+constexpr int GS_ROWS = 8;                       // pixels per chunk
+constexpr int GS_HALF = GS_ROWS * 512;           // one frame's chunk
+constexpr int GS_SLOT = 2 * GS_HALF;
+constexpr int GS_NSLOT = 2;                      // chunks in flight per warp
+constexpr uint64_t GS_WAIT_NS = 1000000000ull;
+
+size_t gumbel_stream_smem_bytes() { return 128 + (size_t)GUMBEL_MAX_TAPS * 256 * 4 + (size_t)GS_WARPS * GS_NSLOT * GS_SLOT; }
+
+template <typename T>
+__global__ void __launch_bounds__(GS_WARPS * 32, 1) gate_pixel_gumbel_stream_kernel(
+    const T* __restrict__ xt, const T* __restrict__ xp, T* __restrict__ xn, const uint8_t* __restrict__ chg_prev,
+    uint8_t* __restrict__ chg_cur, const float* __restrict__ phi, float* __restrict__ taps_out, long long n_pix,
+    int taps, int32_t* __restrict__ count_cur, int32_t* __restrict__ count_next, int* __restrict__ err)
+{
+    constexpr int VX = 16 / (int)sizeof(T), C = 32 * VX;
+    extern __shared__ uint8_t gsm_raw[];
+    uint8_t* gsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(gsm_raw) + 127) & ~(uintptr_t)127);
+    float* sphi = reinterpret_cast<float*>(gsm);                       // [GUMBEL_MAX_TAPS][C]
+    uint8_t* ring = gsm + GUMBEL_MAX_TAPS * 256 * 4;                  // [warp][slot][x_t | x_{t-1}]
+    __shared__ __align__(8) uint64_t full[GS_WARPS][GS_NSLOT];
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        *count_cur = 0;
+        *count_next = 0;
+    }
+    if (threadIdx.x == 0) {
+        for (int w = 0; w < GS_WARPS; ++w)
+            for (int q = 0; q < GS_NSLOT; ++q) ptx::mbar_init(ptx::smem_u32(&full[w][q]), 1);
+        ptx::fence_mbar_init();
+    }
+    for (int i = threadIdx.x; i < GUMBEL_MAX_TAPS * C; i += blockDim.x) sphi[i] = i < taps * C ? phi[i] : 0.f;
+    __syncthreads();
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const long long nch = (n_pix + GS_ROWS - 1) / GS_ROWS;
+    const long long k0 = (long long)blockIdx.x * GS_WARPS + wid, ks = (long long)gridDim.x * GS_WARPS;
+    uint8_t* slots = ring + wid * GS_NSLOT * GS_SLOT;
+    auto issue = [&](long long k, int q) {
+        const long long p0 = k * GS_ROWS;
+        const int np = (int)min((long long)GS_ROWS, n_pix - p0);
+        const uint32_t bytes = (uint32_t)(np * 512);
+        const uint32_t bar = ptx::smem_u32(&full[wid][q]);
+        ptx::mbar_arrive_expect_tx(bar, 2 * bytes);
+        ptx::bulk_load(ptx::smem_u32(slots + q * GS_SLOT), xt + p0 * C, bytes, bar);
+        ptx::bulk_load(ptx::smem_u32(slots + q * GS_SLOT + GS_HALF), xp + p0 * C, bytes, bar);
+    };
+    if (lane == 0)
+        for (int i = 0; i < GS_NSLOT; ++i)
+            if (k0 + i * ks < nch) issue(k0 + i * ks, i);
+    uint32_t phases = 0;
+    int q = 0;
+    for (long long k = k0; k < nch; k += ks) {
+        const long long p0 = k * GS_ROWS;
+        const int np = (int)min((long long)GS_ROWS, n_pix - p0);
+        const uint32_t cprev = lane < np ? chg_prev[p0 + lane] : 0u;   // lanes below np: the chunk's previous flags
+        const uint32_t bar = ptx::smem_u32(&full[wid][q]);
+        const bool ok = __all_sync(0xffffffffu, ptx::mbar_wait(bar, (phases >> q) & 1u, nullptr, err, GS_WAIT_NS)) != 0;
+        if (!ok) {
+            // the copies in flight may still land: wait for them (bounded) before the CTA can exit
+            if (lane == 0)
+                for (int i = 0; i < GS_NSLOT; ++i) {
+                    const int qi = (q + i) % GS_NSLOT;
+                    if (k + i * ks < nch)
+                        ptx::mbar_wait(ptx::smem_u32(&full[wid][qi]), (phases >> qi) & 1u, nullptr, nullptr, GS_WAIT_NS);
+                }
+            return;
+        }
+        const uint4* sx = reinterpret_cast<const uint4*>(slots + q * GS_SLOT);
+        const uint4* sp = reinterpret_cast<const uint4*>(slots + q * GS_SLOT + GS_HALF);
+        float r[GS_ROWS][8];
+        uint32_t chg_rows = 0;   // bit row: the pixel changed
+#pragma unroll
+        for (int row = 0; row < GS_ROWS; ++row) {
+            uint4 av = make_uint4(0, 0, 0, 0), bv = av;
+            if (row < np) {
+                av = sx[row * 32 + lane];
+                bv = sp[row * 32 + lane];
+            }
+            const bool dif = ((av.x ^ bv.x) | (av.y ^ bv.y) | (av.z ^ bv.z) | (av.w ^ bv.w)) != 0u;
+            const bool changed = __any_sync(0xffffffffu, dif);
+            chg_rows |= (changed ? 1u : 0u) << row;
+            const uint32_t cp = __shfl_sync(0xffffffffu, cprev, row);
+            if (row < np && (changed || cp != 0u)) reinterpret_cast<uint4*>(xn + (p0 + row) * C)[lane] = av;
+            float fa[8], fb[8];
+            unpack8(av, fa, (const T*)nullptr);
+            unpack8(bv, fb, (const T*)nullptr);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) r[row][j] = fa[j] - fb[j];
+        }
+        __syncwarp();
+        if (lane == 0 && k + GS_NSLOT * ks < nch) {
+            ptx::fence_proxy_async_smem();   // the slot's reads before the copy that overwrites it
+            issue(k + GS_NSLOT * ks, q);
+        }
+        phases ^= 1u << q;
+        q = q + 1 == GS_NSLOT ? 0 : q + 1;
+        // the chunk's tap products: v[row * 9 + t] = sum over this lane's channels of phi[t][c] r[c]
+        float v[GS_ROWS * GUMBEL_MAX_TAPS];
+#pragma unroll
+        for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) {
+            const float4 w0 = *reinterpret_cast<const float4*>(sphi + t * C + lane * VX);
+            const float4 w1 = VX == 8 ? *reinterpret_cast<const float4*>(sphi + t * C + lane * VX + 4)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int row = 0; row < GS_ROWS; ++row) {
+                float a = w0.x * r[row][0];
+                a = fmaf(w0.y, r[row][1], a);
+                a = fmaf(w0.z, r[row][2], a);
+                a = fmaf(w0.w, r[row][3], a);
+                if (VX == 8) {
+                    a = fmaf(w1.x, r[row][4], a);
+                    a = fmaf(w1.y, r[row][5], a);
+                    a = fmaf(w1.z, r[row][6], a);
+                    a = fmaf(w1.w, r[row][7], a);
+                }
+                v[row * GUMBEL_MAX_TAPS + t] = a;
+            }
+        }
+        // transposed butterfly: each halving exchange keeps half of the rows, until one row's 9 sums are
+        // left in each lane; then plain steps over the remaining lanes of that row
+        static_assert(GS_ROWS == 4 || GS_ROWS == 8, "rows per chunk");
+        constexpr int N1 = GS_ROWS * GUMBEL_MAX_TAPS / 2, N2 = N1 / 2;
+        float v1[N1], v2[N2];
+        {
+            const bool h = (lane >> 4) & 1;
+#pragma unroll
+            for (int i = 0; i < N1; ++i) {
+                const float send = h ? v[i] : v[i + N1], keep = h ? v[i + N1] : v[i];
+                v1[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+            }
+        }
+        {
+            const bool h = (lane >> 3) & 1;
+#pragma unroll
+            for (int i = 0; i < N2; ++i) {
+                const float send = h ? v1[i] : v1[i + N2], keep = h ? v1[i + N2] : v1[i];
+                v2[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+            }
+        }
+        float v3[GUMBEL_MAX_TAPS];
+        int row;
+        if (GS_ROWS == 8) {
+            const bool h = (lane >> 2) & 1;
+#pragma unroll
+            for (int i = 0; i < GUMBEL_MAX_TAPS; ++i) {
+                const float send = h ? v2[i] : v2[(i + GUMBEL_MAX_TAPS) % N2], keep = h ? v2[(i + GUMBEL_MAX_TAPS) % N2] : v2[i];
+                v3[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+            }
+#pragma unroll
+            for (int i = 0; i < GUMBEL_MAX_TAPS; ++i) {
+                v3[i] += __shfl_xor_sync(0xffffffffu, v3[i], 2);
+                v3[i] += __shfl_xor_sync(0xffffffffu, v3[i], 1);
+            }
+            row = (((lane >> 4) & 1) << 2) | (((lane >> 3) & 1) << 1) | ((lane >> 2) & 1);
+        } else {
+#pragma unroll
+            for (int i = 0; i < GUMBEL_MAX_TAPS; ++i) {
+                v3[i] = v2[i % N2];
+                v3[i] += __shfl_xor_sync(0xffffffffu, v3[i], 4);
+                v3[i] += __shfl_xor_sync(0xffffffffu, v3[i], 2);
+                v3[i] += __shfl_xor_sync(0xffffffffu, v3[i], 1);
+            }
+            row = (((lane >> 4) & 1) << 1) | ((lane >> 3) & 1);
+        }
+        // lane holds the 9 sums of pixel `row`; one lane per row writes them
+        if ((lane & (32 / GS_ROWS - 1)) == 0 && row < np) {
+#pragma unroll
+            for (int t = 0; t < GUMBEL_MAX_TAPS; ++t)
+                if (t < taps) taps_out[(p0 + row) * taps + t] = v3[t];
+        }
+        if (lane < np) chg_cur[p0 + lane] = (chg_rows >> lane) & 1u;
+    }
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Gumbel gate, pass 2 of 2: one warp per gate block.  f at an output location
 // is phi_bias plus the partial products of the taps over its receptive field
 // (zero padding: out-of-frame taps add nothing); the block opens when its
@@ -661,6 +845,20 @@ static int gumbel_vec_log2g(const Layer& L)
     return lg;
 }
 
+// the streamed form: 512-byte pixels and at most GUMBEL_MAX_TAPS taps
+static bool gumbel_streamed(const Layer& L)
+{
+    return L.p.c_in * L.esize == 512 && L.p.k_h * L.p.k_w <= GUMBEL_MAX_TAPS;
+}
+
+cudaError_t gumbel_prepare(const Layer& L)
+{
+    if (!gumbel_streamed(L)) return cudaSuccess;
+    return L.p.dtype == SKIPCONV_BF16
+               ? ensure_dynamic_smem((const void*)gate_pixel_gumbel_stream_kernel<__nv_bfloat16>, gumbel_stream_smem_bytes())
+               : ensure_dynamic_smem((const void*)gate_pixel_gumbel_stream_kernel<float>, gumbel_stream_smem_bytes());
+}
+
 // phi in shared memory: [taps][c_in]; the vector form pads it to GUMBEL_MAX_TAPS taps (c_in <= 256 there)
 size_t gumbel_smem_bytes(const Layer& L)
 {
@@ -677,6 +875,18 @@ cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const voi
     const int grid = (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
     const size_t smem = gumbel_smem_bytes(L);
     const int taps = L.p.k_h * L.p.k_w;
+    if (gumbel_streamed(L)) {
+        const int sgrid = L.num_sms;
+        if (L.p.dtype == SKIPCONV_BF16)
+            gate_pixel_gumbel_stream_kernel<__nv_bfloat16><<<sgrid, GS_WARPS * 32, gumbel_stream_smem_bytes(), L.stream>>>(
+                (const __nv_bfloat16*)x_t, (const __nv_bfloat16*)x_prev, (__nv_bfloat16*)x_next, chg_prev, chg_cur,
+                L.gphi, L.pix_taps, n_pix, taps, step_count(L), next_count(L), L.err_dev);
+        else
+            gate_pixel_gumbel_stream_kernel<float><<<sgrid, GS_WARPS * 32, gumbel_stream_smem_bytes(), L.stream>>>(
+                (const float*)x_t, (const float*)x_prev, (float*)x_next, chg_prev, chg_cur, L.gphi, L.pix_taps, n_pix,
+                taps, step_count(L), next_count(L), L.err_dev);
+        return cudaGetLastError();
+    }
     const int lg = gumbel_vec_log2g(L);
     if (lg) {
         const long long per_block = 16LL * (32 >> lg);   // pixels per CTA pass (two per lane group)

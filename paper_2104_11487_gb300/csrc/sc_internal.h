@@ -118,6 +118,8 @@ cudaError_t launch_gate_pixels(const Layer& L, const void* x_t, const void* x_pr
 cudaError_t launch_gate_blocks(const Layer& L, int force);
 // The Gumbel gate's two passes (Eq. 8): per-pixel tap products, then per-block f and threshold
 size_t gumbel_smem_bytes(const Layer& L);
+// Shared-memory limits of the Gumbel passes (at create)
+cudaError_t gumbel_prepare(const Layer& L);
 cudaError_t launch_gate_pixels_gumbel(const Layer& L, const void* x_t, const void* x_prev, void* x_next,
                                       const uint8_t* chg_prev, uint8_t* chg_cur);
 cudaError_t launch_gate_blocks_gumbel(const Layer& L, int force);

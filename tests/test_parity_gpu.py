@@ -175,8 +175,10 @@ GUMBEL_CASES = [
     ("bf16_b8", 1, 48, 40, 64, 64, 1, 8, "bf16"),
     ("f32_b1", 1, 32, 24, 32, 32, 1, 1, "f32"),
     ("f32_stride2_ragged", 2, 37, 29, 16, 24, 2, 4, "f32"),
-    # 32 lanes per pixel in the vector form; and a pixel that is not whole 16-byte vectors (scalar form)
-    ("bf16_c256_b8", 1, 24, 32, 256, 32, 1, 8, "bf16"),
+    # 512-byte pixels (the streamed form; a ragged last chunk of 8 pixels), and a pixel that is not whole
+    # 16-byte vectors (scalar form)
+    ("bf16_c256_b8", 1, 23, 21, 256, 32, 1, 8, "bf16"),
+    ("f32_c128_b4", 2, 19, 17, 128, 16, 1, 4, "f32"),
     ("bf16_c12_b2", 1, 20, 18, 12, 16, 1, 2, "bf16"),
 ]
 
