@@ -700,19 +700,45 @@ __global__ void __launch_bounds__(256) gate_block_gumbel_kernel(const float* __r
             const int bh = min(g.b, g.Ho - by * g.b), bw = min(g.b, g.Wo - bx * g.b);
             const int fy0 = by * g.b * g.stride - g.pad, fx0 = bx * g.b * g.stride - g.pad;
             float best = -INFINITY;
-            for (int q = lane; q < bh * bw; q += 32) {
-                const int i = q / bw, j = q - (q / bw) * bw;
-                float f = phi_bias;
-                for (int kh = 0; kh < g.KH; ++kh) {
-                    const int yy = fy0 + i * g.stride + kh;
-                    if (yy < 0 || yy >= g.H) continue;
-                    for (int kw = 0; kw < g.KW; ++kw) {
-                        const int xx = fx0 + j * g.stride + kw;
-                        if (xx < 0 || xx >= g.W) continue;
-                        f += __ldcg(Tn + ((size_t)yy * g.W + xx) * taps + kh * g.KW + kw);
+            if (g.KH == 3 && g.KW == 3 && bh * bw <= 64) {
+                // 3x3: a lane's (up to) two outputs issue all 18 loads before summing (out-of-frame taps add
+                // 0, which leaves the sum as skipping them would)
+                float t[2][9];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int q = lane + 32 * u;
+                    const bool on = q < bh * bw;
+                    const int i = on ? q / bw : 0, j = on ? q - (q / bw) * bw : 0;
+#pragma unroll
+                    for (int kk = 0; kk < 9; ++kk) {
+                        const int yy = fy0 + i * g.stride + kk / 3, xx = fx0 + j * g.stride + kk % 3;
+                        const bool in = on && yy >= 0 && yy < g.H && xx >= 0 && xx < g.W;
+                        t[u][kk] = in ? __ldcg(Tn + ((size_t)yy * g.W + xx) * 9 + kk) : 0.f;
                     }
                 }
-                best = fmaxf(best, f);
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (lane + 32 * u >= bh * bw) continue;
+                    float f = phi_bias;
+#pragma unroll
+                    for (int kk = 0; kk < 9; ++kk) f += t[u][kk];
+                    best = fmaxf(best, f);
+                }
+            } else {
+                for (int q = lane; q < bh * bw; q += 32) {
+                    const int i = q / bw, j = q - (q / bw) * bw;
+                    float f = phi_bias;
+                    for (int kh = 0; kh < g.KH; ++kh) {
+                        const int yy = fy0 + i * g.stride + kh;
+                        if (yy < 0 || yy >= g.H) continue;
+                        for (int kw = 0; kw < g.KW; ++kw) {
+                            const int xx = fx0 + j * g.stride + kw;
+                            if (xx < 0 || xx >= g.W) continue;
+                            f += __ldcg(Tn + ((size_t)yy * g.W + xx) * taps + kh * g.KW + kw);
+                        }
+                    }
+                    best = fmaxf(best, f);
+                }
             }
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
