@@ -82,6 +82,13 @@ def test_host_side_validation_without_gpu():
     # NULL handles
     assert L.skipconv_step(None, None, None) == _lib.SKIPCONV_ERR_INVALID
     assert L.skipconv_reset_state(None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_step_host(None, None, None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_step_host_async(None, None, None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_sync(None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_step_warped(None, None, None, None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_link_inputs(None, None, None) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_selftest_timeout(None, 1000) == _lib.SKIPCONV_ERR_INVALID
+    assert L.skipconv_check_device(None) == _lib.SKIPCONV_ERR_INVALID
     assert L.skipconv_destroy(None) == _lib.SKIPCONV_OK
 
 
