@@ -179,11 +179,12 @@ def algorithmic(density_active_blocks, changed_pixels, macs_per_block):
 
 
 def flush_l2(buf):
-    if buf is None:            # --no-flush: every step reads more than the L2 holds
-        return
     """Evict L2 between timed steps: write a buffer twice the L2 size, then
     read it back, so that the write-back of dirty lines (the flush's own and
-    the previous step's) happens here rather than inside the next timed step."""
+    the previous step's) happens here rather than inside the next timed step.
+    buf None (--no-flush): every step reads more than the L2 holds anyway."""
+    if buf is None:
+        return
     buf.zero_()
     buf.view(-1, 4096).amax(dim=1)
 

@@ -1,0 +1,28 @@
+"""The benchmark's arithmetic, on the CPU: the algorithmic bytes and FLOPs of
+a c4 step (both frames read in full, the commit of changed pixels, the fp32
+z read-modify-write of the open blocks, the weights; 2 FLOPs per MAC of the
+open blocks), the roofline time they give, and the replica aggregation."""
+import bench
+
+
+def test_algorithmic_bytes_and_flops_of_a_c4_step():
+    x = 8 * 128 * 128 * 256 * 2                     # one bf16 frame of the 8 streams
+    z_block = 8 * 8 * 256 * 4                         # fp32 z of one 8x8 block
+    w = 256 * 256 * 3 * 3 * 2
+    macs = 8 * 8 * 256 * 256 * 3 * 3
+    for active, changed in ((0, 0), (208, 7488), (2048, 131072)):
+        b, f, g = bench.algorithmic(active, changed, macs)
+        assert b == 2 * x + changed * 512 + 2 * active * z_block + w
+        assert g == 2 * x + changed * 512
+        assert f == 2.0 * macs * active
+    # the 10 % step the bench times: 166.49 MB and 15.70 GFLOP, a 24.9 us roofline at the measured peaks
+    b, f, _ = bench.algorithmic(208, 7488, macs)
+    assert abs(b / 1e6 - 166.49) < 0.01 and abs(f / 1e9 - 15.70) < 0.01
+    t_roof = max(f / (1926.3e12), b / (6691.1e9))
+    assert abs(t_roof * 1e6 - 24.88) < 0.01
+
+
+def test_replica_value_counts_every_rank():
+    # stream-frames per second of the whole job: 8 streams per step on every rank
+    assert abs(bench.replica_value(1, 30, 1.5) - 8 * 30 / 1.5e-3) < 1e-6
+    assert abs(bench.replica_value(4, 30, 1.5) - 4 * 8 * 30 / 1.5e-3) < 1e-6
