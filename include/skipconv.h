@@ -150,9 +150,11 @@ SKIPCONV_API int skipconv_step(skipconv_handle h, const void* x_t, const void* s
  * flow: device float32 [n][h][w][2], (dy, dx) in pixels, 4-byte aligned.  A
  * key frame has no previous frame to warp and is the plain key-frame step.
  * Every location of z (and y) moves; the gate, list and x_{t-1} <- x_t are as
- * in skipconv_step.  The first warped step allocates a copy of z.  Errors as
- * skipconv_step, and UNSUPPORTED unless the layer runs the one-launch
- * CUDA-core step and keeps the frame size. */
+ * in skipconv_step.  The first warped step allocates a second z buffer (the
+ * warp writes it and it becomes z, so the pointer skipconv_get_z returns
+ * changes at every warped step) and, where the staged form runs, an fp32
+ * frame for T(x_{t-1}).  Errors as skipconv_step, and UNSUPPORTED unless the
+ * layer runs the one-launch CUDA-core step and keeps the frame size. */
 SKIPCONV_API int skipconv_step_warped(skipconv_handle h, const void* x_t, const void* shortcut, const float* flow);
 
 /* Stack propagation: the input of layer l+1 changes only where layer l's
