@@ -287,11 +287,12 @@ SKIPCONV_API int skipconv_profile_read(skipconv_handle h, long long* launches, d
  * process whose device memory is held by a caching allocator (cudaMalloc may
  * fail there, or force the cache to shrink) and latency-bound callers that
  * cannot take the device-wide synchronisation of cudaMalloc/cudaFree.  It
- * needs no handle.  It computes, for r = x_t - x_prev (Eq. 2), the l1 norm of
- * r over each output location's c_in x k_h x k_w support (Eq. 5, stride and
- * zero padding as in params), its maximum over each b x b block (Sec. 3.2),
- * and opens the blocks above the threshold of params->gate (INPUT_MEAN or
- * INPUT_SUM; dense_mode = 1 opens every block).  The convolution fields of
+ * needs no handle.  It computes the same block gate as skipconv_step: for the
+ * difference r = x_t - x_prev, the sum of |r| over each output location's
+ * c_in x k_h x k_w receptive field (stride and zero padding as in params),
+ * the maximum of that sum over each b x b block of output locations, and opens
+ * the blocks whose maximum exceeds the threshold of params->gate (INPUT_MEAN
+ * or INPUT_SUM; dense_mode = 1 opens every block).  The convolution fields of
  * params are validated as for skipconv_create and otherwise unused.
  *   x_t, x_prev  : device frames [n][h][w][c_in] in dtype (read only)
  *   block_mask   : device uint8 [n][nby][nbx], written

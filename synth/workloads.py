@@ -9,7 +9,15 @@ c4  single 3x3 layer, 256->256, 8 streams of 128x128, T=32, bf16, 8x8 blocks,
     eps 0.05, with a per-frame changed-block density d
 
 Seeds are 1000*config + stream.  Every dimension can be scaled down through
-``make_workload(..., scale=...)`` style overrides for the small parity cases.
+keyword overrides for the small parity cases.
+
+Redraws.  A gate decision whose score lies within a hair of eps is decided by
+rounding, so the parity tests need inputs that keep every gate score away from
+eps.  ``redraw=r`` draws the frames from seed base + REDRAW_STRIDE * r instead
+of the base seed (weights keep their seed); ``MARGIN_REDRAWS`` records, per
+workload at its stated size, the first redraw index whose inputs keep the
+margin (a CPU test recomputes it with the oracle).  This module only draws: it
+does not compute gate scores.
 """
 from __future__ import annotations
 
@@ -21,6 +29,16 @@ from .video import (block_perturbation_video, he_weights, moving_rect_video,
                     moving_squares_video, round_to_bf16, traffic_video)
 
 ACT_NONE, ACT_RELU, ACT_SILU = 0, 1, 2
+
+REDRAW_STRIDE = 100000
+# First redraw index whose frames keep every gate score at least 2e-5 (relative)
+# away from eps, for each workload at its stated size (the margin test in
+# tests/ recomputes these with the oracle and checks that every lower index fails).
+MARGIN_REDRAWS = {"c0": 0, "c1": 0, "c2": 1, "c3": 0, "c4": 0}
+
+
+def _seed(base: int, redraw: int) -> int:
+    return base + REDRAW_STRIDE * int(redraw)
 
 
 @dataclass
@@ -69,16 +87,17 @@ def _weights(seed: int, layers, bf16: bool, bias_std: float):
     return ws, bs
 
 
-def c0(T: int = 8, h: int = 64, w: int = 64, c: int = 32) -> Workload:
+def c0(T: int = 8, h: int = 64, w: int = 64, c: int = 32, redraw: int = 0) -> Workload:
     layers = [LayerDef(c, c, 3, 1, 1, 1, 1, 0.05, name="conv3x3")]
-    frames = moving_squares_video(0, T, h, w, c, n_squares=3, size=8, speed=2, noise_std=0.01)
+    frames = moving_squares_video(_seed(0, redraw), T, h, w, c, n_squares=3, size=8, speed=2, noise_std=0.01)
     ws, bs = _weights(1, layers, bf16=False, bias_std=0.0)
     return Workload("c0", "f32", 1, h, w, c, T, layers, ws, bs, frames[:, None])
 
 
-def c1(T: int = 16, h: int = 128, w: int = 128, c: int = 64, n_squares: int = 6, size: int = 16) -> Workload:
+def c1(T: int = 16, h: int = 128, w: int = 128, c: int = 64, n_squares: int = 6, size: int = 16,
+       redraw: int = 0) -> Workload:
     layers = [LayerDef(c, c, 3, 1, 1, 1, 8, 0.05, name="conv3x3")]
-    frames = round_to_bf16(moving_squares_video(1000, T, h, w, c, n_squares=n_squares, size=size,
+    frames = round_to_bf16(moving_squares_video(_seed(1000, redraw), T, h, w, c, n_squares=n_squares, size=size,
                                                 speed=2, noise_std=0.01))
     ws, bs = _weights(1001, layers, bf16=True, bias_std=0.0)
     return Workload("c1", "bf16", 1, h, w, c, T, layers, ws, bs, frames[:, None])
@@ -96,9 +115,9 @@ def c2_layers(block: int = 4, eps: float = 0.05, width: int = 32, stem: int = 64
     return L
 
 
-def c2(T: int = 32, h: int = 256, w: int = 192, n_blocks: int = 4) -> Workload:
+def c2(T: int = 32, h: int = 256, w: int = 192, n_blocks: int = 4, redraw: int = 0) -> Workload:
     layers = c2_layers(n_blocks=n_blocks)
-    frames = round_to_bf16(moving_rect_video(2000, T, h, w, 3, n_rects=2, rh=48, rw=32, speed=2, jitter=1))
+    frames = round_to_bf16(moving_rect_video(_seed(2000, redraw), T, h, w, 3, n_rects=2, rh=48, rw=32, speed=2, jitter=1))
     ws, bs = _weights(2001, layers, bf16=True, bias_std=0.01)
     return Workload("c2", "bf16", 1, h, w, 3, T, layers, ws, bs, frames[:, None])
 
@@ -113,10 +132,10 @@ def c3_layers(block: int = 8, eps: float = 0.03, c: int = 40, expand: int = 240,
     return L
 
 
-def c3(T: int = 32, n_blocks: int = 3) -> Workload:
+def c3(T: int = 32, n_blocks: int = 3, redraw: int = 0) -> Workload:
     """512x512x3 traffic-like video, 8x8 average-pooled to 64x64x3 and lifted
     to 40 channels by a fixed seeded 1x1 map (input preparation, untimed)."""
-    raw = traffic_video(3000, T)
+    raw = traffic_video(_seed(3000, redraw), T)
     pooled = raw.reshape(T, 64, 8, 64, 8, 3).mean(axis=(2, 4), dtype=np.float64).astype(np.float32)
     rng = np.random.default_rng(3002)
     lift = (rng.standard_normal((3, 40)) / np.sqrt(3.0)).astype(np.float32)
@@ -130,13 +149,13 @@ C4_DENSITIES = (0.0, 0.01, 0.05, 0.10, 0.25, 0.50, 1.00)
 
 
 def c4(density: float = 0.10, T: int = 32, n: int = 8, h: int = 128, w: int = 128, c: int = 256,
-       block: int = 8, dtype: str = "bf16", stream_offset: int = 0) -> Workload:
+       block: int = 8, dtype: str = "bf16", stream_offset: int = 0, redraw: int = 0) -> Workload:
     """Density sweep layer.  `frames` is an iterable yielding (t, frame);
     `stream_offset` selects other streams' seeds (independent replicas)."""
     layers = [LayerDef(c, c, 3, 1, 1, 1, block, 0.05, name="conv3x3")]
     n_changed = int(round(density * (h // block) * (w // block)))
     bf16 = dtype == "bf16"
-    frames = block_perturbation_video(4000, T, n, h, w, c, block, n_changed, bf16=bf16,
+    frames = block_perturbation_video(_seed(4000, redraw), T, n, h, w, c, block, n_changed, bf16=bf16,
                                       stream_offset=stream_offset)
     ws, bs = _weights(4001, layers, bf16=bf16, bias_std=0.0)
     return Workload("c4", dtype, n, h, w, c, T, layers, ws, bs, frames)
@@ -159,4 +178,8 @@ WORKLOADS = {"c0": c0, "c1": c1, "c2": c2, "c3": c3, "c4": c4, "dw3": dw3}
 
 
 def make_workload(name: str, **kw) -> Workload:
+    """The named workload.  Without an explicit ``redraw``, the workloads that
+    record one in MARGIN_REDRAWS use it."""
+    if "redraw" not in kw and name in MARGIN_REDRAWS:
+        kw["redraw"] = MARGIN_REDRAWS[name]
     return WORKLOADS[name](**kw)

@@ -4,7 +4,11 @@ seeded frames and compare them at every frame.
 Comparison rules (floating point decides the gate, so both sides' decisions
 are compared where they are unique):
   * block mask: bit-exact, except blocks whose oracle block score lies within
-    1e-5 relative of eps (an fp32 score there may fall on either side);
+    1e-5 relative of eps (an fp32 score there may fall on either side); for the
+    Gumbel gate (Eq. 8), whose threshold sits at 0, except blocks whose
+    decision is not fixed within the fp32 error bound of f (tests/margin.py);
+    the inputs keep a margin of twice that band, so no block is excluded
+    (run_single_layer and run_stack_teacher_forced assert it);
   * active list: as a set (atomics make the order unspecified), equal to the
     GPU's own mask and to the oracle's mask outside the excluded blocks;
   * z: max-abs error <= 1e-4 for fp32 layers, <= 2e-2 * RMS(z_oracle) for bf16
@@ -16,7 +20,8 @@ from __future__ import annotations
 
 import numpy as np
 
-EPS_BAND = 1e-5
+from margin import EPS_BAND, block_max, gumbel_bound, gumbel_undecided, norm_band  # noqa: F401
+
 TOL_F32_ABS = 1e-4
 TOL_BF16_REL_RMS = 2e-2
 
@@ -29,31 +34,24 @@ def to_device(a: np.ndarray, dtype: str):
     return t.cuda().contiguous()
 
 
-def block_max(score: np.ndarray, b: int) -> np.ndarray:
-    n, ho, wo = score.shape
-    nby, nbx = -(-ho // b), -(-wo // b)
-    pad = np.full((n, nby * b, nbx * b), -np.inf)
-    pad[:, :ho, :wo] = score
-    return pad.reshape(n, nby, b, nbx, b).max(axis=(2, 4))
-
-
 class Compare:
     """Accumulates per-frame comparison results of one layer."""
 
-    def __init__(self, spec, dtype: str, name: str = "", abs_band: float = 0.0):
+    def __init__(self, spec, dtype: str, name: str = ""):
         self.spec, self.dtype, self.name = spec, dtype, name
-        self.abs_band = abs_band      # absolute exclusion band (threshold 0: the Gumbel gate)
         self.excluded = np.zeros((spec.n, spec.nby, spec.nbx), bool)
         self.max_err = 0.0
         self.max_rel = 0.0
         self.frames = 0
         self.n_excluded_events = 0
 
-    def frame(self, t, score, mask_ref, gpu_mask, gpu_list, gpu_count, z_ref, z_gpu, forced):
+    def frame(self, t, score, mask_ref, gpu_mask, gpu_list, gpu_count, z_ref, z_gpu, forced, band=None):
+        """band: the blocks excluded from the mask comparison at this frame; by
+        default those whose oracle block score lies within EPS_BAND of eps."""
         s = self.spec
         if not forced:
-            bmax = block_max(score, s.block)
-            band = np.abs(bmax - s.eps) <= max(EPS_BAND * max(s.eps, 1e-30), self.abs_band)
+            if band is None:
+                band = norm_band(s, score, EPS_BAND)
             self.n_excluded_events += int(band.sum())
             self.excluded |= band
         else:
@@ -96,7 +94,7 @@ def gpu_layer(spec, w, bias, dtype, act=0, emit_y=False, dense_mode=False, conv_
 
 def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0, check_prev=True, name="",
                      reset_at=(), emit_y=False, expect_fused=None, key_interval=0, ref_reset_at=(), phi=None,
-                     phi_bias=0.0):
+                     phi_bias=0.0, max_excluded=0):
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record and the conv path used.
     expect_fused: None, or the info.fused value the layer must report (0 separate
@@ -108,7 +106,7 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
     ref = oracle.OracleLayer(spec, w, bias, dense_mode=dense_mode, phi=phi, phi_bias=phi_bias)
     gl = gpu_layer(spec, w, bias, dtype, dense_mode=dense_mode, conv_path=conv_path, emit_y=emit_y,
                    key_interval=key_interval, phi=phi, phi_bias=phi_bias)
-    cmp = Compare(spec, dtype, name, abs_band=1e-4 if spec.gate == oracle.GATE_GUMBEL else 0.0)
+    cmp = Compare(spec, dtype, name)
     try:
         if expect_fused is not None:
             assert gl.info.fused == int(expect_fused), "%s: fused=%d" % (name, gl.info.fused)
@@ -119,12 +117,17 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
             if t in ref_reset_at:
                 ref.reset()
             forced = ref.key or dense_mode
+            band = None
+            if spec.gate == oracle.GATE_GUMBEL and not forced:
+                r = np.asarray(f, np.float64) - ref.x_prev
+                band = gumbel_undecided(spec, oracle.gumbel_scores(spec, r, phi, phi_bias),
+                                        gumbel_bound(spec, r, phi, phi_bias), spec.eps)
             score, mask_ref = ref.step(f)
             xt = to_device(f, dtype)
             gl.step(xt)
             mask, lst, cnt = gl.gate()
             cmp.frame(t, score, mask_ref, mask.cpu().numpy(), lst.cpu().numpy(), cnt, ref.z,
-                      gl.z().cpu().numpy().astype(np.float64), forced)
+                      gl.z().cpu().numpy().astype(np.float64), forced, band)
             if emit_y:
                 y_gpu = gl.y().float().cpu().numpy().astype(np.float64)
                 y_ref = oracle.layer_output(ref.z, None, 0, 2 if dtype == "bf16" else 1)
@@ -137,14 +140,17 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
                                    xt.view(torch.int16 if dtype == "bf16" else torch.int32)), \
                     "%s t=%d: x_{t-1} is not x_t after the step" % (name, t)
         assert gl.info.conv_path in (1, 2)
+        assert cmp.n_excluded_events <= max_excluded, "%s: %d block decisions in the eps band" % (
+            name, cmp.n_excluded_events)
         return cmp, gl.info.conv_path
     finally:
         gl.close()
 
 
-def run_stack_teacher_forced(wl, T=None, conv_path=0):
+def run_stack_teacher_forced(wl, T=None, conv_path=0, max_excluded=0):
     """Run every layer of a stack workload teacher-forced: each CUDA layer
-    gets the oracle's input sequence (and shortcut) for that layer."""
+    gets the oracle's input sequence (and shortcut) for that layer.  At most
+    max_excluded block decisions (all layers) may fall in the band."""
     import oracle
     from oracle import LayerSpec
     frames = wl.frames if T is None else wl.frames[:T]
@@ -183,6 +189,8 @@ def run_stack_teacher_forced(wl, T=None, conv_path=0):
                 assert not bad.any(), "%s t=%d: %d y values beyond tolerance (max err %.3g, rms %.3g)" % (
                     cmps[li].name, t, int(bad.sum()), float(np.abs(y_gpu - y_ref).max()), rms)
                 stack.append(y_ref)
+        excl = sum(c.n_excluded_events for c in cmps)
+        assert excl <= max_excluded, "%s: %d block decisions in the eps band" % (wl.name, excl)
         return cmps, [g.info.conv_path for g in gls]
     finally:
         for g in gls:

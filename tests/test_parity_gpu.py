@@ -119,6 +119,19 @@ def test_c4_density_small(density, path):
     assert cmp.frames == 32
 
 
+@pytest.mark.parametrize("density", [0.1, 0.5])
+@pytest.mark.parametrize("path", [AUTO, SEPARATE])
+def test_c4_c256_small_every_slice(density, path):
+    """The headline layer's channel counts (256 -> 256) at a small frame size
+    (2 streams of 32x40), 32 frames: on the tensor-core paths every open block
+    is the sum of 4 input-channel slices x 2 output-channel slices, added into
+    z~ by TMA reduce-add, and the full z~ is compared every frame."""
+    wl = synth.make_workload("c4", density=density, T=32, n=2, h=32, w=40, c=256)
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                                 conv_path=path, name="c4-c256 d=%g" % density, expect_fused=FUSED[path])
+    assert used == TENSOR_CORE and cmp.frames == 32
+
+
 @pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_ragged_tail_and_several_tiles(path):
     """Frame sizes that are not multiples of the block (ragged edge blocks)."""
@@ -171,33 +184,43 @@ def test_key_interval_resets_like_the_oracle(path):
 
 
 GUMBEL_CASES = [
-    # name, n, h, w, c_in, c_out, stride, block, dtype
-    ("bf16_b8", 1, 48, 40, 64, 64, 1, 8, "bf16"),
-    ("f32_b1", 1, 32, 24, 32, 32, 1, 1, "f32"),
-    ("f32_stride2_ragged", 2, 37, 29, 16, 24, 2, 4, "f32"),
+    # name, n, h, w, c_in, c_out, stride, block, dtype, redraw (the first frame seed whose gate decisions
+    # all keep twice the fp32 error bound of f away from the threshold, tests/margin.py)
+    ("bf16_b8", 1, 48, 40, 64, 64, 1, 8, "bf16", 0),
+    ("f32_b1", 1, 32, 24, 32, 32, 1, 1, "f32", 0),
+    ("f32_stride2_ragged", 2, 37, 29, 16, 24, 2, 4, "f32", 0),
     # 512-byte pixels (the streamed form; a ragged last chunk of 8 pixels), and a pixel that is not whole
     # 16-byte vectors (scalar form)
-    ("bf16_c256_b8", 1, 23, 21, 256, 32, 1, 8, "bf16"),
-    ("f32_c128_b4", 2, 19, 17, 128, 16, 1, 4, "f32"),
-    ("bf16_c12_b2", 1, 20, 18, 12, 16, 1, 2, "bf16"),
+    ("bf16_c256_b8", 1, 23, 21, 256, 32, 1, 8, "bf16", 0),
+    ("f32_c128_b4", 2, 19, 17, 128, 16, 1, 4, "f32", 0),
+    ("bf16_c12_b2", 1, 20, 18, 12, 16, 1, 2, "bf16", 1),
 ]
+
+
+def gumbel_case_inputs(case):
+    """Frames, layer weights and phi of a Gumbel case (phi random, one output channel)."""
+    name, n, h, w, c_in, c_out, stride, block, dtype, redraw = case
+    rng = np.random.default_rng(400 + block)
+    v = np.stack([synth.moving_squares_video(41 + s + synth.REDRAW_STRIDE * redraw, 5, h, w, c_in, n_squares=2,
+                                             size=8, speed=3, noise_std=0.01) for s in range(n)], axis=1)
+    frames = synth.round_to_bf16(v) if dtype == "bf16" else v.astype(np.float32)
+    wts = synth.he_weights(rng, c_out, c_in, 3, bf16=dtype == "bf16")
+    phi = (rng.standard_normal((c_in, 3, 3)) * 0.2).astype(np.float32)
+    return frames, wts, phi
 
 
 @pytest.mark.parametrize("case", GUMBEL_CASES, ids=[c[0] for c in GUMBEL_CASES])
 @pytest.mark.parametrize("path", [AUTO, CUDA_CORE])
 def test_gumbel_gate(case, path):
     """Gumbel gate at inference (Eq. 8): f(r; phi) > 0 with a random one-output-
-    channel phi and a negative bias, so that small residuals stay closed."""
+    channel phi and a negative bias, so that small residuals stay closed.  No
+    block decision lies within the fp32 error bound of f (asserted by the
+    harness)."""
     from oracle import GATE_GUMBEL
-    name, n, h, w, c_in, c_out, stride, block, dtype = case
+    name, n, h, w, c_in, c_out, stride, block, dtype, _ = case
     if path == AUTO and stride != 1 and dtype == "bf16":
         pytest.skip("covered by the CUDA-core case")
-    rng = np.random.default_rng(400 + block)
-    v = np.stack([synth.moving_squares_video(41 + s, 5, h, w, c_in, n_squares=2, size=8, speed=3, noise_std=0.01)
-                  for s in range(n)], axis=1)
-    frames = synth.round_to_bf16(v) if dtype == "bf16" else v.astype(np.float32)
-    wts = synth.he_weights(rng, c_out, c_in, 3, bf16=dtype == "bf16")
-    phi = (rng.standard_normal((c_in, 3, 3)) * 0.2).astype(np.float32)
+    frames, wts, phi = gumbel_case_inputs(case)
     spec = LayerSpec(n=n, c_in=c_in, c_out=c_out, h=h, w=w, k=3, stride=stride, pad=1, block=block, eps=0.0,
                      gate=GATE_GUMBEL)
     cmp, _ = run_single_layer(spec, wts, None, [frames[t] for t in range(5)], dtype, conv_path=path,
@@ -235,12 +258,24 @@ def test_zero_residual_keeps_state_bitwise():
         gl.close()
 
 
-@pytest.mark.parametrize("path", [AUTO, SEPARATE])
+def test_c4_full_size_full_z():
+    """The bench's workload in the bench's launch configuration (8 streams of
+    128x128x256, 8x8 blocks, 10% block density, the one cooperative fused
+    launch per step), 32 frames: full masks, lists and the full z~ against the
+    full oracle at every frame (Eq. 3), so that every K-slice and output slice
+    of every open block is checked where it lands."""
+    wl = synth.make_workload("c4", density=0.10, T=32)
+    cmp, used = run_single_layer(spec_of(wl), wl.weights[0], wl.biases[0], frames_of(wl), "bf16",
+                                 conv_path=AUTO, name="c4-full", expect_fused=1, check_prev=True)
+    assert used == TENSOR_CORE and cmp.frames == 32
+
+
+@pytest.mark.parametrize("path", [SEPARATE])
 def test_c4_full_size_sampled(path):
-    """The bench's configuration (8 streams of 128x128x256, 8x8 blocks, 10%
-    block density, 32 frames; AUTO is the bench's fused launch): full masks
-    and lists every frame, z at sampled locations (the oracle keeps only
-    those)."""
+    """The bench's workload on the separate launches (8 streams of
+    128x128x256, 8x8 blocks, 10% block density, 32 frames): full masks and
+    lists every frame, z at sampled locations (the oracle keeps only those);
+    the fused launch has the full-z test above."""
     import oracle
     from harness import gpu_layer
     wl = synth.make_workload("c4", density=0.10, T=32)

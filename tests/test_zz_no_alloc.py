@@ -1,10 +1,12 @@
 """skipconv_gate_noalloc (the allocation-free gate entry point) against the
-gate that skipconv_step computes, through the C ABI, on two steps in a row.
+oracle's block gate and against the gate that skipconv_step computes, through
+the C ABI, on two steps in a row.
 
 The file name sorts last so that this test also runs after every other GPU
 test in one session; it passes alone as well.  Masks and open-block sets must
-agree bit for bit, except blocks whose fp64 oracle score lies within 1e-5
-relative of the threshold (an fp32 sum there may fall on either side).
+agree bit for bit with the oracle's, except blocks whose fp64 oracle score
+lies within 1e-5 relative of the threshold (an fp32 sum there may fall on
+either side; the inputs keep twice that margin, so there are none).
 """
 from __future__ import annotations
 
@@ -74,7 +76,11 @@ def test_noalloc_gate_matches_step_gate(case):
         score = oracle.gate_scores(spec, frames[t].astype(np.float64) - frames[t - 1].astype(np.float64))
         sum_score = score * (c * k * k) if gate == GATE_MEAN else score
         band = np.abs(block_max(sum_score, block) - thr) <= EPS_BAND * thr
+        assert not band.any(), "%s t=%d: %d blocks in the eps band" % (name, t, int(band.sum()))
         ok = ~band
+        m_oracle = oracle.block_gate(spec, score)
+        assert np.array_equal(m_new[ok], m_oracle[ok]), "%s t=%d: masks differ from the oracle's" % (name, t)
+        assert np.array_equal(ids, np.flatnonzero(m_oracle.ravel())), "%s t=%d: open set != oracle's" % (name, t)
         assert np.array_equal(m_new[ok], m_ref[ok]), "%s t=%d: masks differ" % (name, t)
         assert set(np.unique(m_new)) <= {0, 1}
         assert np.array_equal(ids, np.flatnonzero(m_new.ravel())), "%s t=%d: list != mask" % (name, t)
