@@ -16,4 +16,4 @@ from .video import (  # noqa: F401
     block_perturbation_video,
     he_weights,
 )
-from .workloads import WORKLOADS, LayerDef, Workload, make_workload  # noqa: F401
+from .workloads import MARGIN_REDRAWS, REDRAW_STRIDE, WORKLOADS, LayerDef, Workload, make_workload  # noqa: F401
