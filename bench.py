@@ -71,6 +71,10 @@ def parse():
     ap.add_argument("--no-soak", action="store_true",
                     help="skip the untimed steps around the timed region (for profiler runs)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-table", action="store_true",
+                    help="skip the oracle's per-workload table (every config, all cores and one)")
+    ap.add_argument("--cpu-table-seconds", type=float, default=1.5,
+                    help="seconds of oracle work per row of the per-workload table")
     ap.add_argument("--clocks-log", default=None, metavar="PATH",
                     help="keep the nvidia-smi samples of the timed region in this CSV (default: a temporary file)")
     return ap.parse_args()
@@ -589,6 +593,98 @@ def cpu_oracle_sample(seconds, density, max_frames=200):
                       "double-precision C loops" % (done, t_total)}
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu / /proc/cpuinfo), else the machine type."""
+    import platform
+    import subprocess
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return platform.machine()
+
+
+def cpu_workload_sample(name, seconds, threads):
+    """The oracle stepping a whole workload (every layer of a stack) on the
+    host cores: the key frame untimed on all cores, then frames 1, 2, ... timed
+    with `threads` threads until `seconds` of work (at least one frame) or the
+    end of the video."""
+    import oracle
+    import synth
+    wl = synth.make_workload(name)
+    refs, shortcuts = [], []
+    h, w = wl.h, wl.w
+    for li, L in enumerate(wl.layers):
+        spec = oracle.LayerSpec(n=wl.n, c_in=L.c_in, c_out=L.c_out, h=h, w=w, k=L.k, stride=L.stride, pad=L.pad,
+                                groups=L.groups, block=L.block, eps=L.eps)
+        refs.append(oracle.OracleLayer(spec, wl.weights[li], wl.biases[li]))
+        h, w = spec.ho, spec.wo
+    round_mode = 2 if wl.dtype == "bf16" else 1
+
+    def frame(x):
+        stack = [np.asarray(x, np.float64)]
+        for li, L in enumerate(wl.layers):
+            refs[li].step(stack[-1])
+            if len(wl.layers) > 1:
+                sc = None if L.shortcut < 0 else stack[L.shortcut]
+                stack.append(oracle.layer_output(refs[li].z, sc, L.act, round_mode))
+
+    cores = oracle.num_threads()
+    frame(wl.frames[0])
+    oracle.set_num_threads(threads)
+    done, t_total = 0, 0.0
+    try:
+        for t in range(1, wl.T):
+            t0 = time.perf_counter()
+            frame(wl.frames[t])
+            t_total += time.perf_counter() - t0
+            done += 1
+            if t_total >= seconds:
+                break
+    finally:
+        oracle.set_num_threads(cores)
+    return {"frames_per_s": wl.n * done / t_total, "ms_per_frame": t_total / done * 1e3, "threads": threads,
+            "sample": "frames 1-%d after the key frame (%d layers)" % (done, len(wl.layers))}
+
+
+def cpu_baseline_table(seconds_each):
+    """The oracle on every workload, at all host cores and at one: c0-c3 as
+    whole stacks (frames/s) and the c4 layer at each sweep density (stream 0,
+    stream-frames/s).  One core takes c4 only up to 10 % density: a single
+    frame at 50 % is about 10 GFLOP of double-precision loops."""
+    import oracle
+    cores = oracle.num_threads()
+    rows = []
+    for name in ("c0", "c1", "c2", "c3"):
+        for threads in (cores, 1):
+            r = cpu_workload_sample(name, seconds_each, threads)
+            r["workload"] = name
+            rows.append(r)
+    from synth.workloads import C4_DENSITIES
+    for d in C4_DENSITIES:
+        for threads in (cores, 1):
+            if threads == 1 and d > 0.10:
+                continue
+            oracle.set_num_threads(threads)
+            try:
+                r = cpu_oracle_sample(seconds_each, d, max_frames=60)
+            finally:
+                oracle.set_num_threads(cores)
+            rows.append({"workload": "c4 d=%g" % d, "frames_per_s": r["value"], "ms_per_frame": 1e3 / r["value"],
+                         "threads": threads, "sample": r["sample"]})
+    return {"cpu": cpu_model(), "cores": cores, "seconds_per_sample": seconds_each,
+            "unit": "frames/s (c4: stream-frames/s of stream 0)", "rows": rows}
+
+
 # ------------------------------------------------------------- ranks
 class Ranks:
     """Process-group plumbing of a replica run (torchrun, one rank per GPU):
@@ -833,6 +929,8 @@ def main():
         one = cpu_oracle_sample(args.cpu_seconds / 3, args.density)
         oracle.set_num_threads(cores)
         line["cpu_baseline"]["single_core"] = {"value": one["value"], "unit": one["unit"], "sample": one["sample"]}
+        if not args.no_cpu_table:
+            line["cpu_baseline"]["per_workload"] = cpu_baseline_table(args.cpu_table_seconds)
     layer.close()
     if args.drift and rank == 0:
         line["drift_vs_dense"] = drift_report(torch)

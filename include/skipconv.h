@@ -82,8 +82,10 @@ typedef enum { SKIPCONV_ACT_NONE = 0, SKIPCONV_ACT_RELU = 1, SKIPCONV_ACT_SILU =
 typedef enum {
     SKIPCONV_PATH_AUTO = 0,        /* tensor cores where supported, else CUDA cores;
                                       layers whose dense step is at most 2^26 MACs
-                                      run the one-launch CUDA-core step (a step of
-                                      that size is latency-bound)                 */
+                                      run the one-launch step, a CTA per tile of
+                                      gate blocks (a step of that size is latency-
+                                      bound), with its contraction on the tensor
+                                      cores for dense (groups = 1) bf16 layers    */
     SKIPCONV_PATH_CUDA_CORE = 1,   /* float32 FMA direct convolution              */
     SKIPCONV_PATH_TENSOR_CORE = 2, /* tcgen05 implicit GEMM (bf16 in, fp32 accum)  */
     SKIPCONV_PATH_TENSOR_CORE_SEPARATE = 3, /* the same convolution, but never fused with
@@ -228,14 +230,16 @@ SKIPCONV_API int skipconv_get_gate(skipconv_handle h, const uint8_t** block_mask
 typedef struct {
     int ho, wo;        /* output frame size                                   */
     int nby, nbx;      /* gate blocks per stream                              */
-    int conv_path;     /* path actually used: SKIPCONV_PATH_CUDA_CORE or _TENSOR_CORE */
+    int conv_path;     /* where the contraction runs: SKIPCONV_PATH_CUDA_CORE or
+                          SKIPCONV_PATH_TENSOR_CORE                           */
     int num_sms;       /* SMs of the device the handle lives on               */
     size_t state_bytes;/* device bytes held by the handle                     */
     int fused;         /* 0: separate launches (gate passes, convolution, y);
                           1: each step is one cooperative tensor-core launch
                           (gate and convolution pipelined over the streams);
-                          2: each step is one CUDA-core launch, a CTA per tile
-                          of gate blocks working from its own input footprint */
+                          2: each step is one launch, a CTA per tile of gate
+                          blocks working from its own input footprint (its
+                          contraction on tcgen05 where conv_path says so)     */
 } skipconv_info;
 SKIPCONV_API int skipconv_get_info(skipconv_handle h, skipconv_info* info);
 

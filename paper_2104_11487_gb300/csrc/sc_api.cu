@@ -279,9 +279,15 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
     }
     const bool want_cc = L.p.conv_path == SKIPCONV_PATH_CUDA_CORE ||
                          L.p.conv_path == SKIPCONV_PATH_CUDA_CORE_SEPARATE;
-    // AUTO: small layers (latency-bound steps) take the one-launch CUDA-core step
+    // AUTO: small layers (latency-bound steps) take the one-launch step, a CTA per tile of gate
+    // blocks; its contraction runs on the tensor cores for dense bf16 layers (depthwise and fp32
+    // layers keep the CUDA cores)
     const bool small = L.p.conv_path == SKIPCONV_PATH_AUTO && step_local_preferred(L);
     L.path = (want_cc || small || !tc_ok) ? SKIPCONV_PATH_CUDA_CORE : SKIPCONV_PATH_TENSOR_CORE;
+    L.local_tc = (L.p.conv_path == SKIPCONV_PATH_AUTO && L.path == SKIPCONV_PATH_CUDA_CORE &&
+                  L.p.dtype == SKIPCONV_BF16 && L.p.groups == 1 && !(L.cpg == 1 && L.opg == 1))
+                     ? 1
+                     : 0;
     L.ci_pad = ((L.p.c_in + 63) / 64) * 64;
     L.co_pad = ((L.p.c_out + 127) / 128) * 128;
 
@@ -795,7 +801,7 @@ int skipconv_get_info(skipconv_handle h, skipconv_info* info)
     info->wo = L->wo;
     info->nby = L->nby;
     info->nbx = L->nbx;
-    info->conv_path = L->path;
+    info->conv_path = (L->fused == 2 && L->local_tc) ? SKIPCONV_PATH_TENSOR_CORE : L->path;
     info->fused = L->fused;
     info->num_sms = L->num_sms;
     info->state_bytes = L->state_bytes;

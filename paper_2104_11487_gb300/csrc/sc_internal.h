@@ -87,6 +87,7 @@ struct Layer {
 
     // one-launch CUDA-core step (sc_step_local.cu)
     int local_staged;       // 1: its TMA-footprint / staged-weight form
+    int local_tc;           // 1: the staged form's contraction runs on the tensor cores (tcgen05)
     CUtensorMap tmap_fp[2]; // footprint boxes of the two state frames
     CUtensorMap tmap_ztile; // tile boxes of z
     void* w_loc;            // weights packed per CTA slice, layer dtype

@@ -1,4 +1,5 @@
-// One-launch Skip-Conv step for layers on the CUDA-core path.
+// One-launch Skip-Conv step for small (latency-bound) layers and for layers on
+// the CUDA-core path.
 //
 // Every CTA takes a tile of sb x sb gate blocks and does the whole step for
 // it from its own input footprint (the union of the receptive fields of the
@@ -12,10 +13,13 @@
 //      k_h x k_w receptive field (the local support norm of Eq. 5), the block
 //      maximum (max-pooling of the gate, Sec. 3.2) against the threshold;
 //   4. the open blocks appended to the compact list (one atomic per tile);
-//   5. w * r_t at the open locations, added into z in place (Eq. 3), from the
-//      shared-memory residual: a register-blocked contraction over
-//      k_h*k_w*(c_in/groups) on float32 FMAs (dense and grouped layers), or
-//      one thread per channel and location (depthwise);
+//   5. w * r_t at the open locations, added into z in place (Eq. 3): for dense
+//      bf16 layers under SKIPCONV_PATH_AUTO a tcgen05 implicit GEMM of the
+//      open locations' receptive fields (A, built in shared memory from the
+//      footprints) by the slice's weights (B), accumulated in tensor memory;
+//      otherwise from the shared-memory residual, a register-blocked
+//      contraction over k_h*k_w*(c_in/groups) on float32 FMAs (dense and
+//      grouped layers), or one thread per channel and location (depthwise);
 //   6. y = act(z) at the open locations, or y = act(z + shortcut) over the
 //      whole tile when the layer has a shortcut.
 // Halo pixels shared with neighbouring tiles are recomputed instead of
@@ -39,6 +43,7 @@
 
 #include "sc_internal.h"
 #include "sc_ptx.cuh"
+#include "sc_tc_common.cuh"
 
 namespace sc {
 namespace {
@@ -452,7 +457,10 @@ struct FastArgs {
     int force;
     int n, H, W, C, Ho, Wo, Co, KH, KW, stride, pad, b, nby, nbx, act;
     int sb, nty, ntx, FH, FW, CP, nsl, K;
+    int Kp;                    // tensor-core contraction: K rounded up to 16 (the MMA's K step)
     uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq;   // byte offsets
+    uint32_t off_a;            // tensor-core contraction: the A region (its last 2 KB stay free)
+    int aregion;               //   and its size in bytes
     float thr;
     // stack propagation
     const uint8_t* px_chg;       // the layer that produced x_t: its per-block "y may have changed" flags
@@ -530,15 +538,38 @@ __device__ __forceinline__ float2 load_pair(const __nv_bfloat16* p)
     return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
 }
 
-template <typename T, bool DW, int SW, bool WP>
+// Eight fp32 values as eight bf16 (round to nearest even), in memory order.
+__device__ __forceinline__ uint4 pack_bf16x8(const float4& a, const float4& b)
+{
+    uint4 v;
+    __nv_bfloat162 h[4] = {__floats2bfloat162_rn(a.x, a.y), __floats2bfloat162_rn(a.z, a.w),
+                           __floats2bfloat162_rn(b.x, b.y), __floats2bfloat162_rn(b.z, b.w)};
+    v.x = *reinterpret_cast<uint32_t*>(&h[0]);
+    v.y = *reinterpret_cast<uint32_t*>(&h[1]);
+    v.z = *reinterpret_cast<uint32_t*>(&h[2]);
+    v.w = *reinterpret_cast<uint32_t*>(&h[3]);
+    return v;
+}
+
+constexpr int TC_ROWS = 128;                // MMA rows (open locations) per pass
+constexpr int TC_MAX_KG = 9 * 256 / 8;      // k-groups of w in the offset table (3x3, 256 channels)
+// The plain step's A: [x_t | -x_{t-1}] (exact in bf16, each half against w) when true; else
+// r = x_t - x_{t-1} rounded to bf16 (one half).
+constexpr bool TC_EXACT = true;
+constexpr int TC_AREGION_MAX = 32 * 1024;   // most shared memory for A (its last 2 KB stay free)
+
+template <typename T, bool DW, int SW, bool WP, bool TC>
 __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_constant__ CUtensorMap tm_xt,
                                                                const __grid_constant__ CUtensorMap tm_xp,
                                                                const __grid_constant__ CUtensorMap tm_z,
                                                                const __grid_constant__ CUtensorMap tm_sc,
                                                                const FastArgs a)
 {
+    static_assert(!TC || (!DW && sizeof(T) == 2), "the tensor-core contraction takes dense bf16 layers");
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[3];    // 0: weights, 1: footprints, 2: z (and shortcut) tile
+    // 0: weights, 1: footprints, 2: z (and shortcut) tile, 3-4: MMAs done reading A buffer 0 / 1
+    __shared__ __align__(8) uint64_t bars[5];
+    __shared__ uint32_t s_tmem;
     __shared__ int s_open[MAX_TILE_BLOCKS];
     __shared__ int s_max[MAX_TILE_BLOCKS];      // per gate block: largest support sum (float bits)
     __shared__ int s_nloc;
@@ -576,6 +607,10 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         mbar_init(bar_w, 1);
         mbar_init(bar_x, 1);
         mbar_init(bar_z, 1);
+        if (TC) {
+            mbar_init(smem_u32(&bars[3]), 1);
+            mbar_init(smem_u32(&bars[4]), 1);
+        }
         fence_mbar_init();
         // the weights are constant state: fetch them before waiting for the producer of x_t
         mbar_arrive_expect_tx(bar_w, a.wbytes);
@@ -586,6 +621,20 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         s_tchg = 0;
     }
     if (tid < MAX_TILE_BLOCKS) s_max[tid] = 0;
+    if (TC) {
+        // the accumulator's 32 TMEM columns, taken while the previous grid finishes.  The grid that
+        // launched this one early had every CTA take its columns before it let this grid start, and
+        // a grid after this one starts only once every CTA here passed the dependency wait, so at
+        // most two grids hold columns on an SM: at most 8 CTAs of 256 threads, 256 of 512 columns,
+        // and an allocation here never waits for a CTA that waits for this grid.
+        if (warp == 0) {
+            tmem_alloc(smem_u32(&s_tmem), 32);
+            tmem_relinquish();
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
     grid_dependency_wait();
     if (blockIdx.x == 0 && tid == 0) *a.count_next = 0;
     // owned input pixels of this tile (every input pixel has exactly one owner tile)
@@ -625,6 +674,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
                 }
             }
             if (tid == 0) mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);   // the weight copy in flight
+            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
             return;
         }
     }
@@ -653,6 +703,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             mbar_wait(bar_x, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             if (has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
             return;
         }
     }
@@ -683,7 +734,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             for (int e = 0; e < 8; ++e)
                 if (e < ne) sum += fabsf(r[e]);
             Pp[it] = sum;
-            if (!DW) {
+            if (!DW && (!TC || WP)) {   // the fp32 residual feeds the FMA contraction and the warped step's A
                 float4* rr = reinterpret_cast<float4*>(R + (size_t)q * a.CP + k * EPC);
                 rr[0] = make_float4(r[0], r[1], r[2], r[3]);
                 if (EPC == 8) rr[1] = make_float4(r[4], r[5], r[6], r[7]);
@@ -807,6 +858,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         if (!__syncthreads_and(ok)) {
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             if (any_open || has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
+            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
             return;
         }
     }
@@ -861,6 +913,179 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
                     y[zo + 1] = y1;
                 }
             }
+        }
+    } else if (TC) {
+        // The contraction on the tensor cores (tcgen05, bf16 operands, fp32 accumulation), in
+        // passes of up to 128 open locations: D[m][o] = sum_k A[m][k] B[o][k].  Row m of A is the
+        // m-th open location's receptive field, k = tap * C + ci over K (padded to Kp, a multiple
+        // of 16).  A plain step takes w * r_t as w * x_t + w * (-x_{t-1}) (Eq. 3 is linear in r):
+        // A is [x_t | -x_{t-1}], both halves exact in bf16 and each multiplied by B = w, so the
+        // products are exact and only the fp32 sums round.  A warped step's previous input
+        // T(x_{t-1}) is not bf16: there A is r = x_t - T(x_{t-1}) rounded to bf16 (one half).
+        // B is the slice's weights, staged by the bulk copy.  Both operands use the
+        // no-swizzle K-major layout of core matrices (8 rows x 16 bytes, rows 16 bytes apart, row
+        // groups 128 bytes apart): B as [k/8][SW][8]; A as [k/8][R][8] with R the pass's rows
+        // rounded up to 8, so that A holds only the open locations.  An MMA reads 128 rows: rows
+        // past R fall on the next k-group or on the 2 KB kept free past the A region, and only
+        // feed rows of D that are not read.  A is built in one go where it fits in the region,
+        // else in chunks of k-groups into two buffers (the MMAs of one chunk run while the next
+        // is built).  D: TMEM lane m, columns 0..SW-1 (taken after the dependency wait).
+        const uint32_t tmem = s_tmem;
+        bool ok = true;
+        if (M > 0) {
+            const uint32_t bm0 = smem_u32(&bars[3]), bm1 = smem_u32(&bars[4]);
+            uint8_t* Abuf = base + a.off_a;
+            const uint8_t* Wb = reinterpret_cast<const uint8_t*>(Ws);
+            const int hkg = a.Kp / 8;                                  // k-groups of w (even)
+            const int tkg = (!WP && TC_EXACT) ? 2 * hkg : hkg;         // k-groups of A (even)
+            // per k-group of A (8 consecutive k): its element offset from a row's first footprint
+            // pixel, bit 31 set for x_{t-1}; per row of a pass: that pixel's element offset.  Both in
+            // the k-split scratch, which the tensor-core contraction does not use.
+            const int px = WP ? a.CP : a.C;   // elements per footprint pixel of A's source
+            int* koff = reinterpret_cast<int*>(base + a.off_scr);
+            int* rofs = koff + TC_MAX_KG;
+            for (int kg = tid; kg < hkg; kg += FT) {
+                const int k = kg * 8;   // a k-group of 8 never straddles two taps: C is a multiple of 8
+                const int tap = k / a.C, ci = k - tap * a.C;
+                const int kh = tap / a.KW, kw = tap - kh * a.KW;
+                koff[kg] = k < a.K ? (kh * a.FW + kw) * px + ci : -1;   // -1: padding past K
+            }
+            constexpr uint32_t idesc = idesc_bf16_f32(TC_ROWS, SW);
+            uint32_t phase = 0u;   // bit b: the next phase to wait for on buffer b's barrier
+            uint32_t pend = 0u;    // bit b: MMAs reading buffer b were committed and not yet waited for
+            // wait for the MMAs that read buffer b (bounded; the error word records a timeout)
+            auto drain = [&](int b) {
+                if (pend & (1u << b)) {
+                    ok = mbar_wait(b ? bm1 : bm0, (phase >> b) & 1u, nullptr, a.err, LOCAL_WAIT_NS) && ok;
+                    phase ^= 1u << b;
+                    pend &= ~(1u << b);
+                }
+            };
+            for (int m0 = 0; m0 < M && ok; m0 += TC_ROWS) {
+                const int mr = min(TC_ROWS, M - m0);
+                const int rb = ((mr + 7) & ~7) * 16;                       // bytes of one k-group of A
+                const int usable = a.aregion - 2048;
+                // k-groups per chunk: all of them, or (two buffers) an even number that fits half the region
+                const int ckg = tkg * rb <= usable ? tkg : (usable / 2 / rb) & ~1;
+                const int nch = (tkg + ckg - 1) / ckg;
+                for (int m = tid; m < mr; m += FT) {
+                    const int loc = locs[m0 + m], li = loc >> 16, lj = loc & 0xffff;
+                    rofs[m] = (li * a.stride * a.FW + lj * a.stride) * px;
+                }
+                __syncthreads();
+                for (int c = 0; c < nch; ++c) {
+                    const int bs = c & 1;
+                    drain(bs);   // the MMAs that read this buffer two chunks ago
+                    uint8_t* Ab = Abuf + bs * ckg * rb;
+                    const int kg0 = c * ckg, nkg = min(ckg, tkg - kg0);
+                    for (int it = tid; it < nkg * mr; it += FT) {
+                        const int j = it / mr, m = it - j * mr;
+                        const int kg = kg0 + j, prev = kg >= hkg;
+                        const int ko = koff[prev ? kg - hkg : kg];
+                        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+                        if (ko >= 0) {
+                            const int e = rofs[m] + ko;
+                            if (WP) {
+                                const float4* src = reinterpret_cast<const float4*>(R + e);
+                                v = pack_bf16x8(src[0], src[1]);
+                            } else if (TC_EXACT) {
+                                v = *reinterpret_cast<const uint4*>((prev ? Xp : Xt) + e);
+                                if (prev) {   // -x_{t-1}: the sign bits of the eight bf16 values, exactly
+                                    v.x ^= 0x80008000u;
+                                    v.y ^= 0x80008000u;
+                                    v.z ^= 0x80008000u;
+                                    v.w ^= 0x80008000u;
+                                }
+                            } else {
+                                v = bf16x8_sub(*reinterpret_cast<const uint4*>(Xt + e),
+                                               *reinterpret_cast<const uint4*>(Xp + e));
+                            }
+                        }
+                        *reinterpret_cast<uint4*>(Ab + j * rb + m * 16) = v;
+                    }
+                    fence_proxy_async_smem();
+                    ok = __syncthreads_and(ok) != 0;
+                    if (!ok) break;
+                    if (warp == 0) {
+                        tc_fence_after();
+                        if (elect_one()) {
+                            for (int j = 0; j < nkg; j += 2) {
+                                const uint64_t ad = smem_desc(smem_u32(Ab + j * rb), rb, 128, 0);
+                                const int wg = kg0 + j < hkg ? kg0 + j : kg0 + j - hkg;   // both halves of A take w
+                                const uint64_t bd = smem_desc(smem_u32(Wb + (size_t)wg * SW * 16), SW * 16, 128, 0);
+                                mma_bf16(tmem, ad, bd, idesc, (kg0 + j) != 0 ? 1u : 0u);
+                            }
+                            mma_commit(bs ? bm1 : bm0);
+                        }
+                        __syncwarp();
+                    }
+                    pend |= 1u << bs;
+                }
+                // the last commit covers every MMA issued before it; both buffers' phases advance
+                drain(0);
+                drain(1);
+                ok = __syncthreads_and(ok) != 0;
+                if (!ok) break;
+                tc_fence_after();
+                // D -> shared memory (the A region, free once the MMAs completed), rows SW + 4 floats
+                // apart so that the row-per-thread writes spread over the banks; then every thread
+                // takes (location, 4 channels) items: z~ += D, y = act(z~ [+ shortcut])
+                constexpr int DS = SW + 4;
+                float* Dst = reinterpret_cast<float*>(Abuf);
+                if (tid < TC_ROWS) {
+                    // warp w reads TMEM lanes 32w .. 32w + 31: thread = row = open location m0 + tid
+                    const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+                    uint32_t v[SW];
+                    if constexpr (SW == 32) tmem_ld_32x32b_x32(taddr, v);
+                    else tmem_ld_32x32b_x16(taddr, v);
+                    tmem_wait_ld();
+                    if (tid < mr) {
+                        float4* drow = reinterpret_cast<float4*>(Dst + tid * DS);
+#pragma unroll
+                        for (int q = 0; q < SW / 4; ++q)
+                            drow[q] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                                  __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+                    }
+                }
+                tc_fence_before();
+                __syncthreads();
+                {
+                    const int nq = min(SW, a.Co - o_base) / 4;   // c_out is a multiple of 4
+                    for (int it = tid; it < mr * nq; it += FT) {
+                        const int m = it / nq, q = it - m * nq;
+                        const int loc = locs[m0 + m], li = loc >> 16, lj = loc & 0xffff;
+                        const int lz = li * span + lj;
+                        const size_t zo = (((size_t)nn * a.Ho + oy0 + li) * a.Wo + ox0 + lj) * a.Co + o_base + 4 * q;
+                        const float4 d = reinterpret_cast<const float4*>(Dst + m * DS)[q];
+                        const float4 zt = reinterpret_cast<const float4*>(Zs + lz * ZW)[q];
+                        float u[4] = {zt.x + d.x, zt.y + d.y, zt.z + d.z, zt.w + d.w};
+                        *reinterpret_cast<float4*>(a.z + zo) = make_float4(u[0], u[1], u[2], u[3]);
+                        if (y) {
+                            const int zi = lz * ZW + 4 * q;
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) u[e] = activate(has_sc ? u[e] + to_f32(Ss[zi + e]) : u[e], a.act);
+                            const __nv_bfloat162 lo = __floats2bfloat162_rn(u[0], u[1]), hi = __floats2bfloat162_rn(u[2], u[3]);
+                            uint2 pk;
+                            pk.x = *reinterpret_cast<const uint32_t*>(&lo);
+                            pk.y = *reinterpret_cast<const uint32_t*>(&hi);
+                            *reinterpret_cast<uint2*>(y + zo) = pk;
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncthreads();   // D is read before the next pass writes it
+            }
+            if (!ok) {
+                // an MMA never completed (a wait ran out and set the error word): give the ones in
+                // flight a last bounded wait before the columns go back
+                if (pend & 1u) mbar_wait(bm0, phase & 1u, nullptr, nullptr, LOCAL_WAIT_NS);
+                if (pend & 2u) mbar_wait(bm1, (phase >> 1) & 1u, nullptr, nullptr, LOCAL_WAIT_NS);
+                __syncthreads();
+            }
+        }
+        if (warp == 0) {
+            tc_fence_after();
+            tmem_dealloc(tmem, 32);
         }
     } else {
         constexpr int NQ = SW / 4;
@@ -1002,6 +1227,25 @@ __global__ void pack_local_weights_kernel(const float* __restrict__ wcc, T* __re
     }
 }
 
+// Weights of the tensor-core contraction: per slice, [Kp/8][sw][8] bf16 (the
+// no-swizzle K-major layout of the MMA's B operand), element (k, n) = w(k, o)
+// with o = slice * sw + n, k = tap * c_in + ci; zero for k >= K and o >= c_out.
+__global__ void pack_local_tc_weights_kernel(const float* __restrict__ wcc, __nv_bfloat16* __restrict__ out, int K,
+                                             int Kp, int Co, int nsl, int sw)
+{
+    const long long total = (long long)nsl * Kp * sw;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int e = (int)(i % 8);
+        long long rest = i / 8;
+        const int n = (int)(rest % sw);
+        rest /= sw;
+        const int g = (int)(rest % (Kp / 8)), sl = (int)(rest / (Kp / 8));
+        const int k = g * 8 + e, o = sl * sw + n;
+        out[i] = __float2bfloat16_rn(o < Co && k < K ? wcc[(size_t)k * Co + o] : 0.f);
+    }
+}
+
 struct LocalShape {
     int sb, span, FH, FW, CP;
     size_t smem;
@@ -1048,9 +1292,11 @@ struct StagedShape {
     int sw;          // output channels per CTA (dense layers)
     int nsl;
     int zw;          // channels of the z / shortcut tile boxes
+    int Kp;          // tensor-core contraction: K rounded up to 16 (else K)
     size_t own_max;  // most input pixels a tile owns
     uint32_t wbytes;
-    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq;
+    uint32_t off_xp, off_w, off_r, off_p, off_loc, off_scr, off_z, off_sc, off_chg, off_dq, off_a;
+    int aregion;     // tensor-core contraction: bytes for A (all of it in one go where that fits)
     size_t smem;
 };
 
@@ -1066,11 +1312,14 @@ StagedShape staged_shape(const Layer& L, int sb, bool wp = false)
     const bool dw = is_depthwise(L);
     const size_t fp = (size_t)t.g.FH * t.g.FW;
     const int K = L.p.k_h * L.p.k_w * L.p.c_in;
+    const bool tc = L.local_tc && !dw;
     // small tiles with few output channels: narrower slices spread an open tile over more SMs
     t.sw = (t.g.span <= 4 && L.p.c_out <= 32) ? SW_NARROW : SW_WIDE;
     t.nsl = dw ? 1 : (L.p.c_out + t.sw - 1) / t.sw;
     t.zw = dw ? L.p.c_out : t.sw;
-    const size_t wb = dw ? (size_t)L.p.k_h * L.p.k_w * L.p.c_in * L.esize : (size_t)K * t.sw * L.esize;
+    // the tensor-core contraction's weights: [K/8][sw][8] bf16, K padded to the MMA's K step
+    t.Kp = tc ? (K + 15) / 16 * 16 : K;
+    const size_t wb = dw ? (size_t)L.p.k_h * L.p.k_w * L.p.c_in * L.esize : (size_t)t.Kp * t.sw * L.esize;
     t.wbytes = (uint32_t)((wb + 15) & ~(size_t)15);
     // largest owned input region of a tile (the last tile row / column owns the rest of the frame)
     const int span_in = t.g.span * L.p.stride;
@@ -1085,17 +1334,30 @@ StagedShape staged_shape(const Layer& L, int sb, bool wp = false)
     t.off_xp = xb;
     t.off_w = xb + pb;
     t.off_r = t.off_w + up128(t.wbytes);
-    t.off_p = t.off_r + (dw ? 0 : up128(fp * t.g.CP * sizeof(float)));
+    // the fp32 residual: the FMA contraction's and the warped tensor-core step's operand
+    t.off_p = t.off_r + ((dw || (tc && !wp)) ? 0 : up128(fp * t.g.CP * sizeof(float)));
     t.off_loc = t.off_p + up128(fp * sizeof(float));
     t.off_scr = t.off_loc + up128((size_t)t.g.span * t.g.span * sizeof(int));
     // scratch: the footprint pass's chunk partials, later (dense) the k-split partial sums
     const size_t chunks = fp * (L.p.c_in * L.esize / 16);
-    const size_t scr = std::max(chunks * (sizeof(float) + 1), dw ? (size_t)0 : (size_t)FT * FLPI * 4 * sizeof(float));
+    // (the tensor-core contraction keeps its k-group and row offset tables there instead)
+    const size_t scr = std::max(chunks * (sizeof(float) + 1),
+                                dw ? (size_t)0
+                                   : tc ? (size_t)(TC_MAX_KG + TC_ROWS) * sizeof(int)
+                                        : (size_t)FT * FLPI * 4 * sizeof(float));
     t.off_z = t.off_scr + up128(scr);
     t.off_sc = t.off_z + up128(tile_elems * sizeof(float));
     t.off_chg = t.off_sc + (L.p.emit_y ? up128(tile_elems * L.esize) : 0);
     t.off_dq = t.off_chg + up128(t.own_max);
-    t.smem = (size_t)t.off_dq + up128(fp) + 1024;
+    t.off_a = t.off_dq + up128(fp);
+    // A for a whole pass of the tile's locations (at most 128 rows) in one go, plus the 2 KB an MMA may
+    // read past it, where that fits TC_AREGION_MAX; else TC_AREGION_MAX, built in chunks
+    const size_t a_rows = (size_t)std::min(128, t.g.span * t.g.span);
+    const size_t a_kg = (size_t)(t.Kp / 8) * ((TC_EXACT && !wp) ? 2 : 1);
+    const size_t a_need = a_kg * ((a_rows + 7) / 8 * 8) * 16 + 2048;
+    const size_t d_need = ((a_rows + 7) / 8 * 8) * (size_t)(t.sw + 4) * sizeof(float);   // D staged for the epilogue
+    t.aregion = tc ? (int)up128(std::max(std::min(a_need, (size_t)TC_AREGION_MAX), d_need)) : 0;
+    t.smem = (size_t)t.off_a + t.aregion + 1024;
     return t;
 }
 
@@ -1154,15 +1416,24 @@ bool encode_tile_map(CUtensorMap* m, const void* base, const Layer& L, const Sta
 template <typename T, bool WP>
 const void* staged_kernel_of(const Layer& L, int sw)
 {
-    if (is_depthwise(L)) return (const void*)step_local_staged_kernel<T, true, SW_WIDE, WP>;
-    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<T, false, SW_NARROW, WP>
-                           : (const void*)step_local_staged_kernel<T, false, SW_WIDE, WP>;
+    if (is_depthwise(L)) return (const void*)step_local_staged_kernel<T, true, SW_WIDE, WP, false>;
+    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<T, false, SW_NARROW, WP, false>
+                           : (const void*)step_local_staged_kernel<T, false, SW_WIDE, WP, false>;
+}
+
+template <bool WP>
+const void* staged_tc_kernel_of(int sw)
+{
+    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<__nv_bfloat16, false, SW_NARROW, WP, true>
+                           : (const void*)step_local_staged_kernel<__nv_bfloat16, false, SW_WIDE, WP, true>;
 }
 
 const void* staged_kernel_of(const Layer& L, int sw, bool wp = false)
 {
-    if (L.p.dtype == SKIPCONV_BF16)
+    if (L.p.dtype == SKIPCONV_BF16) {
+        if (L.local_tc) return wp ? staged_tc_kernel_of<true>(sw) : staged_tc_kernel_of<false>(sw);
         return wp ? staged_kernel_of<__nv_bfloat16, true>(L, sw) : staged_kernel_of<__nv_bfloat16, false>(L, sw);
+    }
     return wp ? staged_kernel_of<float, true>(L, sw) : staged_kernel_of<float, false>(L, sw);
 }
 
@@ -1357,8 +1628,11 @@ cudaError_t launch_staged(Layer& L, const StagedShape& t, const void* x_t, const
     a.nty = (L.nby + t.g.sb - 1) / t.g.sb;
     a.ntx = (L.nbx + t.g.sb - 1) / t.g.sb;
     a.FH = t.g.FH; a.FW = t.g.FW; a.CP = t.g.CP; a.nsl = t.nsl; a.K = L.p.k_h * L.p.k_w * L.p.c_in;
+    a.Kp = t.Kp;
     a.off_xp = t.off_xp; a.off_w = t.off_w; a.off_r = t.off_r; a.off_p = t.off_p; a.off_loc = t.off_loc;
     a.off_scr = t.off_scr; a.off_z = t.off_z; a.off_sc = t.off_sc; a.off_chg = t.off_chg; a.off_dq = t.off_dq;
+    a.off_a = t.off_a;
+    a.aregion = t.aregion;
     a.thr = L.gate_thr;
     a.px_chg = px ? px->ychg : nullptr;
     a.pxb = px ? px->p.block : 1; a.pxnby = px ? px->nby : 1; a.pxnbx = px ? px->nbx : 1;
@@ -1419,6 +1693,11 @@ static cudaError_t alloc_ychg(Layer& L)
 cudaError_t step_local_prepare(Layer& L)
 {
     StagedShape t;
+    // the tensor-core contraction needs the staged form (and room for its A region), and its k-group
+    // offset table holds TC_MAX_KG entries
+    if (L.local_tc && (L.p.dtype != SKIPCONV_BF16 || is_depthwise(L) || L.p.groups != 1 ||
+                       (L.p.k_h * L.p.k_w * L.p.c_in + 15) / 16 * 2 > TC_MAX_KG || !staged_ok(L, nullptr)))
+        L.local_tc = 0;
     if (staged_ok(L, &t)) {
         if (!encode_footprint_map(&L.tmap_fp[0], L.xbuf[0], L, t) || !encode_footprint_map(&L.tmap_fp[1], L.xbuf[1], L, t) ||
             !encode_tile_map(&L.tmap_ztile, L.z, L, t, true)) {
@@ -1436,9 +1715,12 @@ cudaError_t step_local_prepare(Layer& L)
         if (e != cudaSuccess) return e;
         const bool dw = is_depthwise(L);
         const int K = L.p.k_h * L.p.k_w * L.p.c_in;
-        const long long total = dw ? (long long)K * L.p.c_out : (long long)t.nsl * K * t.sw;
+        const long long total = dw ? (long long)K * L.p.c_out : (long long)t.nsl * t.Kp * t.sw;
         const int grid = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
-        if (L.p.dtype == SKIPCONV_BF16)
+        if (L.local_tc)
+            pack_local_tc_weights_kernel<<<grid, 256, 0, L.stream>>>(L.w_cc, (__nv_bfloat16*)L.w_loc, K, t.Kp,
+                                                                     L.p.c_out, t.nsl, t.sw);
+        else if (L.p.dtype == SKIPCONV_BF16)
             pack_local_weights_kernel<__nv_bfloat16><<<grid, 256, 0, L.stream>>>(
                 L.w_cc, (__nv_bfloat16*)L.w_loc, dw ? L.p.k_h * L.p.k_w : K, L.p.c_out, t.nsl, t.sw, dw ? 1 : 0);
         else
