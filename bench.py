@@ -873,13 +873,47 @@ def main():
             skipconv_step_host_async(layer.handle, host[args.warmup + 1 + i], zh[i % 2])
         skipconv_sync(layer.handle)
         t_e2e = max_over_ranks(time.perf_counter() - t0)
-        line["e2e"] = {"value": replica_value(world, args.steps, t_e2e * 1e3), "unit": UNIT,
-                       "h2d_bytes_per_step": host[0].numel() * 2, "d2h_bytes_per_step": zh[0].numel() * 4,
-                       "call": "skipconv_step_host_async then skipconv_sync (host frame in, full fp32 z out; "
-                               "copies of neighbouring steps overlap)",
+        # the sparse result: each step's open blocks of z (count, ids, values) written by the device straight
+        # into pinned host memory -- what a consumer holding z needs (Eq. 3 changes z only there)
+        from paper_2104_11487_gb300 import skipconv_step_host_sparse_async
+        nblk = N_STREAMS * (H // BLOCK) * (W // BLOCK)
+        zbk = [torch.empty((nblk, BLOCK, BLOCK, C), dtype=torch.float32).pin_memory() for _ in range(2)]
+        lbk = [torch.empty(nblk, dtype=torch.int32).pin_memory() for _ in range(2)]
+        cbk = [torch.zeros(1, dtype=torch.int32).pin_memory() for _ in range(2)]
+        layer.reset()
+        for i in range(args.warmup + 1):
+            skipconv_step_host_sparse_async(layer.handle, host[i], zbk[i % 2], lbk[i % 2], cbk[i % 2])
+        skipconv_sync(layer.handle)
+        barrier()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            skipconv_step_host_sparse_async(layer.handle, host[args.warmup + 1 + i], zbk[i % 2], lbk[i % 2],
+                                            cbk[i % 2])
+        skipconv_sync(layer.handle)
+        t_sparse = max_over_ranks(time.perf_counter() - t0)
+        # bytes the result took over the link: an untimed pass reading each step's count
+        layer.reset()
+        for i in range(args.warmup + 1):
+            skipconv_step_host_sparse_async(layer.handle, host[i], zbk[0], lbk[0], cbk[0])
+        skipconv_sync(layer.handle)
+        cnts = []
+        for i in range(args.steps):
+            skipconv_step_host_sparse_async(layer.handle, host[args.warmup + 1 + i], zbk[0], lbk[0], cbk[0])
+            skipconv_sync(layer.handle)
+            cnts.append(int(cbk[0][0]))
+        d2h_sparse = 4 + statistics.mean(cnts) * (4 + BLOCK * BLOCK * C * 4)
+        line["e2e"] = {"value": replica_value(world, args.steps, t_sparse * 1e3), "unit": UNIT,
+                       "h2d_bytes_per_step": host[0].numel() * 2, "d2h_bytes_per_step": d2h_sparse,
+                       "call": "skipconv_step_host_sparse_async then skipconv_sync (host frame in; the step's open "
+                               "blocks of fp32 z, their ids and count out, written by the device into pinned "
+                               "host memory; uploads of neighbouring steps overlap)",
+                       "full_z_value": replica_value(world, args.steps, t_e2e * 1e3),
+                       "full_z_d2h_bytes_per_step": zh[0].numel() * 4,
+                       "full_z_call": "skipconv_step_host_async then skipconv_sync (host frame in, full fp32 z out; "
+                                      "copies of neighbouring steps overlap)",
                        "sync_value": replica_value(world, args.steps, t_sync * 1e3),
-                       "sync_call": "skipconv_step_host (one synchronous call per step)"}
-        del host
+                       "sync_call": "skipconv_step_host (one synchronous call per step, full z out)"}
+        del host, zbk
 
     # 4) density sweep vs the all-ones dense mode of the same kernels
     if not args.no_sweep:

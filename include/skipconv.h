@@ -171,7 +171,10 @@ SKIPCONV_API int skipconv_step_warped(skipconv_handle h, const void* x_t, const 
  * its residual is zero there, so the full step would keep every block closed
  * and write nothing.  Results are identical to unlinked steps.  Otherwise
  * (another x_t, a producer that stepped twice or not at all, key frames) the
- * step reads the whole frame as usual.  producer_x = NULL removes the links.
+ * step reads the whole frame as usual, and so does a layer whose tiles all fit
+ * on the GPU at once (one wave of CTAs): skipping tiles takes no wave off such
+ * a step, while reading the flags would delay every tile by a memory round
+ * trip.  producer_x = NULL removes the links.
  * Errors: INVALID (NULL handle, self link, shortcut link without x link,
  * shapes, dtypes or streams that do not match), UNSUPPORTED (this layer not on
  * the one-launch CUDA-core step with TMA footprints, or a producer that keeps
@@ -200,6 +203,28 @@ SKIPCONV_API int skipconv_step_host(skipconv_handle h, const void* x_t_host, flo
  * Errors: INVALID (NULL handle or x_t_host), OOM, CUDA; a device error word
  * set by an earlier step is reported as by skipconv_step. */
 SKIPCONV_API int skipconv_step_host_async(skipconv_handle h, const void* x_t_host, float* z_out_host);
+
+/* Pipelined host-buffer step with a sparse result (Eq. 3: z~ changes only at
+ * the open blocks, the rest is copied from the previous step).  x_t_host is
+ * uploaded and the step runs as in skipconv_step_host_async; then, on the
+ * handle's stream, a kernel writes straight into the host buffers (pinned and
+ * mapped into the device's address space, e.g. cudaHostAlloc; every pinned
+ * allocation is mapped on systems with unified addressing):
+ *   *count_host        the number of open blocks of this step;
+ *   list_host[i]       the i-th open block id, (n * nby + by) * nbx + bx
+ *                      (i < count; order unspecified, as skipconv_get_gate);
+ *   z_blocks_host[i]   that block's z~ after the step, float32 [b][b][c_out]
+ *                      (output locations past the frame's edge are 0).
+ * A consumer that holds z~ applies the blocks to keep it equal to the
+ * device's z~; after create, a reset or a key frame every block is open.
+ * The buffers must have room for n*nby*nbx blocks and ids and are lent until
+ * skipconv_sync returns.  Enqueued without waiting; the first call allocates
+ * the two device staging frames of x (no staging of z).  Errors: INVALID
+ * (NULL handle or pointer, or a host buffer the device cannot address), OOM,
+ * CUDA; a device error word set by an earlier step is reported as by
+ * skipconv_step. */
+SKIPCONV_API int skipconv_step_host_sparse_async(skipconv_handle h, const void* x_t_host, float* z_blocks_host,
+                                                 int32_t* list_host, int32_t* count_host);
 
 /* Wait for every step and copy enqueued on the handle's streams; reports the
  * device error word (SKIPCONV_OK, SKIPCONV_ERR_TIMEOUT, SKIPCONV_ERR_DEVICE). */

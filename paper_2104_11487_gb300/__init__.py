@@ -11,4 +11,5 @@ from .skipconv import (SkipConvLayer, device_tensor, skipconv_check_device, skip
                        skipconv_get_stats, skipconv_get_y, skipconv_get_z, skipconv_profile, skipconv_profile_read,
                        skipconv_link_inputs, skipconv_reset_state, skipconv_selftest_timeout,
                        skipconv_set_gate_weights, skipconv_step,
-                       skipconv_step_host, skipconv_step_host_async, skipconv_step_warped, skipconv_sync)
+                       skipconv_step_host, skipconv_step_host_async, skipconv_step_host_sparse_async,
+                       skipconv_step_warped, skipconv_sync)

@@ -29,6 +29,7 @@ SIGNATURES = {
     "skipconv_step": (c_int, [c_void_p, c_void_p, c_void_p]),
     "skipconv_step_host": (c_int, [c_void_p, c_void_p, c_void_p]),
     "skipconv_step_host_async": (c_int, [c_void_p, c_void_p, c_void_p]),
+    "skipconv_step_host_sparse_async": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "skipconv_sync": (c_int, [c_void_p]),
     "skipconv_destroy": (c_int, [c_void_p]),
     "skipconv_get_z": (c_int, [c_void_p, c_void_p]),

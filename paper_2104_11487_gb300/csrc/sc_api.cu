@@ -721,14 +721,53 @@ int skipconv_step_host_async(skipconv_handle h, const void* x_t_host, float* z_o
     return SKIPCONV_OK;
 }
 
+// A pointer into pinned host memory that is mapped into the device's address space, as the device
+// pointer of that same byte; NULL if the memory is not pinned and mapped.
+static void* device_view(void* host)
+{
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, host) != cudaSuccess || at.type != cudaMemoryTypeHost) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    void* dev = nullptr;
+    if (cudaHostGetDevicePointer(&dev, host, 0) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return dev;
+}
+
+int skipconv_step_host_sparse_async(skipconv_handle h, const void* x_t_host, float* z_blocks_host, int32_t* list_host,
+                                    int32_t* count_host)
+{
+    Layer* L = get(h);
+    if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
+    if (!x_t_host || !z_blocks_host || !list_host || !count_host)
+        return set_error("a host buffer is NULL"), SKIPCONV_ERR_INVALID;
+    float* zb = static_cast<float*>(device_view(z_blocks_host));
+    int32_t* lb = static_cast<int32_t*>(device_view(list_host));
+    int32_t* cb = static_cast<int32_t*>(device_view(count_host));
+    if (!zb || !lb || !cb)
+        return set_error("the result buffers must be pinned host memory mapped into the device's address space"),
+               SKIPCONV_ERR_INVALID;
+    // upload and step as the pipelined call does, without the z read-back
+    const int st = skipconv_step_host_async(h, x_t_host, nullptr);
+    if (st) return st;
+    // the step just enqueued used count slot (t - 1) % 2
+    const cudaError_t e = launch_gather_open_blocks(*L, L->counters + ((L->t - 1) & 1), zb, lb, cb);
+    return e == cudaSuccess ? SKIPCONV_OK : status_of(e);
+}
+
 int skipconv_sync(skipconv_handle h)
 {
     Layer* L = get(h);
     if (!L) return set_error("NULL handle"), SKIPCONV_ERR_INVALID;
-    cudaError_t e = cudaSuccess;
-    for (cudaStream_t st : {L->up_stream, L->stream, L->down_stream})
-        if (st && e == cudaSuccess) e = cudaStreamSynchronize(st);
-    if (!L->up_stream && e == cudaSuccess) e = cudaStreamSynchronize(L->stream);
+    // the copy streams exist once a pipelined call ran; the handle's stream may be the legacy default
+    // stream (NULL), which is synchronised all the same
+    cudaError_t e = L->up_stream ? cudaStreamSynchronize(L->up_stream) : cudaSuccess;
+    if (e == cudaSuccess) e = cudaStreamSynchronize(L->stream);
+    if (e == cudaSuccess && L->down_stream) e = cudaStreamSynchronize(L->down_stream);
     if (e != cudaSuccess) return status_of(e);
     return check_device_word(L);
 }

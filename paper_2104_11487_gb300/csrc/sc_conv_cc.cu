@@ -293,6 +293,53 @@ cudaError_t launch_reset_z(const Layer& L)
     return cudaGetLastError();
 }
 
+// Open blocks of z into a packed buffer: CTA j takes blocks j, j + grid, ... of the step's list;
+// each copies the block's b x b x c_out values (16-byte vectors when c_out is a multiple of 4),
+// zeros past the frame's edge.  CTA 0 also copies the count and the list.
+__global__ void gather_open_blocks_kernel(const float* __restrict__ z, const int32_t* __restrict__ list,
+                                          const int32_t* __restrict__ count, float* __restrict__ zb,
+                                          int32_t* __restrict__ list_out, int32_t* __restrict__ count_out, int Ho,
+                                          int Wo, int Co, int b, int nby, int nbx)
+{
+    const int cnt = *count;
+    if (blockIdx.x == 0) {
+        for (int i = threadIdx.x; i < cnt; i += blockDim.x) list_out[i] = list[i];
+        if (threadIdx.x == 0) *count_out = cnt;
+    }
+    const int row = b * Co;   // floats of one block row
+    for (int i = blockIdx.x; i < cnt; i += gridDim.x) {
+        const int id = list[i];
+        const int bx = id % nbx, by = (id / nbx) % nby, n = id / (nbx * nby);
+        float* dst = zb + (size_t)i * b * row;
+        if ((Co & 3) == 0) {
+            const int q4 = row / 4;
+            for (int e = threadIdx.x; e < b * q4; e += blockDim.x) {
+                const int r = e / q4, q = e - r * q4;
+                const int oy = by * b + r, ox = bx * b + (4 * q) / Co;
+                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (oy < Ho && ox < Wo)
+                    v = *reinterpret_cast<const float4*>(z + (((size_t)n * Ho + oy) * Wo + ox) * Co + (4 * q) % Co);
+                reinterpret_cast<float4*>(dst + (size_t)r * row)[q] = v;
+            }
+        } else {
+            for (int e = threadIdx.x; e < b * row; e += blockDim.x) {
+                const int r = e / row, q = e - r * row;
+                const int oy = by * b + r, ox = bx * b + q / Co;
+                dst[e] = (oy < Ho && ox < Wo) ? z[(((size_t)n * Ho + oy) * Wo + ox) * Co + q % Co] : 0.f;
+            }
+        }
+    }
+}
+
+cudaError_t launch_gather_open_blocks(const Layer& L, const int32_t* count, float* zb, int32_t* list_out,
+                                      int32_t* count_out)
+{
+    const int grid = L.num_sms * 4;
+    gather_open_blocks_kernel<<<grid, 256, 0, L.stream>>>(L.z, L.list, count, zb, list_out, count_out, L.ho,
+                                                         L.wo, L.p.c_out, L.p.block, L.nby, L.nbx);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack_weights(Layer& L, const void* w_oihw, double* w_l1_dev)
 {
     const long long total = (long long)L.p.c_out * L.cpg * L.p.k_h * L.p.k_w;

@@ -94,6 +94,7 @@ struct Layer {
     uint8_t* ychg;          // per gate block: the last step may have changed y (layers with y)
     uint8_t* tile_chg;      // [2][tiles]: some owned input pixel's change flag is set in chg[parity]
     int ntiles;             // tiles of the staged form
+    int local_resident;     // CTAs of the staged form that fit on the GPU at once (SMs x CTAs per SM)
 
     // stack propagation (skipconv_link_inputs): the layers whose y this layer takes as x_t and as
     // the shortcut, and their step counts when this layer last stepped
@@ -129,6 +130,10 @@ cudaError_t launch_gate_blocks_gumbel(const Layer& L, int force);
 cudaError_t launch_conv_cc(const Layer& L, const void* x_t, const void* x_prev);
 cudaError_t launch_y_refresh(const Layer& L, const void* shortcut);
 cudaError_t launch_reset_z(const Layer& L);
+// The step's open blocks of z (count, ids, [b][b][c_out] values) into device-addressable buffers
+// (mapped host memory for skipconv_step_host_sparse_async).
+cudaError_t launch_gather_open_blocks(const Layer& L, const int32_t* count, float* zb, int32_t* list_out,
+                                      int32_t* count_out);
 cudaError_t launch_pack_weights(Layer& L, const void* w_oihw, double* w_l1_out);
 
 // Tensor-core convolution (sc_conv_tc.cu)

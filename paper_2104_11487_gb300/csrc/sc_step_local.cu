@@ -1740,6 +1740,11 @@ cudaError_t step_local_prepare(Layer& L)
         e = cudaMemsetAsync(L.tile_chg, 0, 2 * (size_t)L.ntiles, L.stream);
         if (e == cudaSuccess) e = alloc_ychg(L);
         if (e == cudaSuccess) e = ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
+        if (e == cudaSuccess) {
+            int per_sm = 0;
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, staged_kernel_of(L, t.sw), FT, t.smem);
+            L.local_resident = L.num_sms * per_sm;
+        }
         // warped steps run the staged form's warped variant, or the general form when it does not fit
         StagedShape tp, tw;
         if (e == cudaSuccess && staged_wp_ok(L, &tp, &tw)) e = ensure_dynamic_smem(staged_kernel_of(L, tw.sw, true), tw.smem);
@@ -1832,6 +1837,11 @@ cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, i
         return launch_staged(L, tw, x_t, shortcut, force, nullptr, nullptr, &L.tmap_tx, true);
     if (L.local_staged && !flow) {
         if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
+        // Linked inputs pay only where the grid is more than one wave of resident CTAs: skipped tiles
+        // then take whole waves off the step.  Within one wave every tile runs at once, the step lasts
+        // as long as its slowest (open) tile, and the flag read would only delay each tile's footprint
+        // load by a memory round trip; such a step reads the whole frame instead.
+        if ((long long)L.ntiles * t.nsl <= (long long)L.local_resident) px = psc = nullptr;
         return launch_staged(L, t, x_t, shortcut, force, px, psc, &L.tmap_fp[cur], false);
     }
     const LocalShape s = choose_shape(L);

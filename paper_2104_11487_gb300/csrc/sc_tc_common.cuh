@@ -22,7 +22,8 @@ __device__ __forceinline__ void decode_block(int id, int nby, int nbx, int& n, i
     n = id / (nbx * nby);
 }
 
-// Eight bf16 residuals x - p, formed in fp32 and rounded to nearest.
+// Eight bf16 residuals x - p, each the bf16 subtraction rounded to nearest
+// (packed pairs: four instructions for eight values).
 __device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
 {
     const __nv_bfloat162* a = reinterpret_cast<const __nv_bfloat162*>(&x);
@@ -30,11 +31,7 @@ __device__ __forceinline__ uint4 bf16x8_sub(const uint4& x, const uint4& p)
     uint4 out;
     __nv_bfloat162* o = reinterpret_cast<__nv_bfloat162*>(&out);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const float2 fa = __bfloat1622float2(a[k]);
-        const float2 fb = __bfloat1622float2(b[k]);
-        o[k] = __floats2bfloat162_rn(fa.x - fb.x, fa.y - fb.y);
-    }
+    for (int k = 0; k < 4; ++k) o[k] = __hsub2(a[k], b[k]);
     return out;
 }
 

@@ -51,6 +51,12 @@ def skipconv_step_host_async(handle: int, x_t_host, z_out_host=None) -> None:
           _lib.lib().skipconv_step_host_async(handle, _ptr(x_t_host), _ptr(z_out_host)))
 
 
+def skipconv_step_host_sparse_async(handle: int, x_t_host, z_blocks_host, list_host, count_host) -> None:
+    check("skipconv_step_host_sparse_async",
+          _lib.lib().skipconv_step_host_sparse_async(handle, _ptr(x_t_host), _ptr(z_blocks_host), _ptr(list_host),
+                                                     _ptr(count_host)))
+
+
 def skipconv_sync(handle: int) -> None:
     check("skipconv_sync", _lib.lib().skipconv_sync(handle))
 
