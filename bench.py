@@ -259,8 +259,9 @@ def make_layer(wl, torch, dense_mode=False, path="fused", gate="input", key_inte
 
 
 PROFILE_FILES = {"gate_pixel": ("gate_pixel", ("sc_gate.cu",)), "gate_block": ("gate_block", ("sc_gate.cu",)),
-                 "conv": ("conv_ws", ("sc_conv_ws.cu", "sc_ws_roles.cuh")),
-                 "step_fused": ("step_fused", ("sc_step_fused.cu", "sc_ws_roles.cuh"))}
+                 "conv": ("conv_ws", ("sc_conv_ws.cu", "sc_ws_roles.cuh", "sc_tc_common.cuh", "sc_ptx.cuh")),
+                 "step_fused": ("step_fused", ("sc_step_fused.cu", "sc_ws_roles.cuh", "sc_tc_common.cuh",
+                                               "sc_ptx.cuh"))}
 
 
 def source_digest(files):

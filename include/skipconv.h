@@ -171,9 +171,9 @@ SKIPCONV_API int skipconv_step_warped(skipconv_handle h, const void* x_t, const 
  * its residual is zero there, so the full step would keep every block closed
  * and write nothing.  Results are identical to unlinked steps.  Otherwise
  * (another x_t, a producer that stepped twice or not at all, key frames) the
- * step reads the whole frame as usual, and so does a layer whose tiles all fit
- * on the GPU at once (one wave of CTAs): skipping tiles takes no wave off such
- * a step, while reading the flags would delay every tile by a memory round
+ * step reads the whole frame as usual, and so does a layer whose tiles take at
+ * most two waves of resident CTAs: skipping tiles takes no wave off such a
+ * step, while reading the flags would delay every tile by a memory round
  * trip.  producer_x = NULL removes the links.
  * Errors: INVALID (NULL handle, self link, shortcut link without x link,
  * shapes, dtypes or streams that do not match), UNSUPPORTED (this layer not on

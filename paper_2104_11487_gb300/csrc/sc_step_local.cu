@@ -552,6 +552,9 @@ __device__ __forceinline__ uint4 pack_bf16x8(const float4& a, const float4& b)
 }
 
 constexpr int TC_ROWS = 128;                // MMA rows (open locations) per pass
+// TMEM columns of the accumulator: the slice's output channels (a power of 2, at least 32)
+template <int SW>
+constexpr uint32_t tc_cols() { return SW < 32 ? 32u : (uint32_t)SW; }
 constexpr int TC_MAX_KG = 9 * 256 / 8;      // k-groups of w in the offset table (3x3, 256 channels)
 // The plain step's A: [x_t | -x_{t-1}] (exact in bf16, each half against w) when true; else
 // r = x_t - x_{t-1} rounded to bf16 (one half).
@@ -628,7 +631,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         // most two grids hold columns on an SM: at most 8 CTAs of 256 threads, 256 of 512 columns,
         // and an allocation here never waits for a CTA that waits for this grid.
         if (warp == 0) {
-            tmem_alloc(smem_u32(&s_tmem), 32);
+            tmem_alloc(smem_u32(&s_tmem), tc_cols<SW>());
             tmem_relinquish();
         }
         tc_fence_before();
@@ -674,7 +677,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
                 }
             }
             if (tid == 0) mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);   // the weight copy in flight
-            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
+            if (TC && warp == 0) tmem_dealloc(s_tmem, tc_cols<SW>());
             return;
         }
     }
@@ -703,7 +706,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
             mbar_wait(bar_x, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             if (has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
-            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
+            if (TC && warp == 0) tmem_dealloc(s_tmem, tc_cols<SW>());
             return;
         }
     }
@@ -858,7 +861,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         if (!__syncthreads_and(ok)) {
             mbar_wait(bar_w, 0, nullptr, nullptr, LOCAL_WAIT_NS);
             if (any_open || has_sc) mbar_wait(bar_z, 0, nullptr, nullptr, LOCAL_WAIT_NS);
-            if (TC && warp == 0) tmem_dealloc(s_tmem, 32);
+            if (TC && warp == 0) tmem_dealloc(s_tmem, tc_cols<SW>());
             return;
         }
     }
@@ -1033,18 +1036,23 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
                 constexpr int DS = SW + 4;
                 float* Dst = reinterpret_cast<float*>(Abuf);
                 if (tid < TC_ROWS) {
-                    // warp w reads TMEM lanes 32w .. 32w + 31: thread = row = open location m0 + tid
+                    // warp w reads TMEM lanes 32w .. 32w + 31: thread = row = open location m0 + tid,
+                    // 32 columns (16 for a 16-channel slice) at a time
                     const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
-                    uint32_t v[SW];
-                    if constexpr (SW == 32) tmem_ld_32x32b_x32(taddr, v);
-                    else tmem_ld_32x32b_x16(taddr, v);
-                    tmem_wait_ld();
-                    if (tid < mr) {
-                        float4* drow = reinterpret_cast<float4*>(Dst + tid * DS);
+                    constexpr int CC = SW < 32 ? SW : 32;
+#pragma unroll 1
+                    for (int c0 = 0; c0 < SW; c0 += CC) {
+                        uint32_t v[CC];
+                        if constexpr (CC == 32) tmem_ld_32x32b_x32(taddr + c0, v);
+                        else tmem_ld_32x32b_x16(taddr + c0, v);
+                        tmem_wait_ld();
+                        if (tid < mr) {
+                            float4* drow = reinterpret_cast<float4*>(Dst + tid * DS + c0);
 #pragma unroll
-                        for (int q = 0; q < SW / 4; ++q)
-                            drow[q] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                                  __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+                            for (int q = 0; q < CC / 4; ++q)
+                                drow[q] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                                      __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+                        }
                     }
                 }
                 tc_fence_before();
@@ -1085,7 +1093,7 @@ __global__ void __launch_bounds__(FT, 1) step_local_staged_kernel(const __grid_c
         }
         if (warp == 0) {
             tc_fence_after();
-            tmem_dealloc(tmem, 32);
+            tmem_dealloc(tmem, tc_cols<SW>());
         }
     } else {
         constexpr int NQ = SW / 4;
@@ -1313,8 +1321,12 @@ StagedShape staged_shape(const Layer& L, int sb, bool wp = false)
     const size_t fp = (size_t)t.g.FH * t.g.FW;
     const int K = L.p.k_h * L.p.k_w * L.p.c_in;
     const bool tc = L.local_tc && !dw;
-    // small tiles with few output channels: narrower slices spread an open tile over more SMs
-    t.sw = (t.g.span <= 4 && L.p.c_out <= 32) ? SW_NARROW : SW_WIDE;
+    // small tiles with few output channels: narrower slices spread an open tile over more SMs.  A
+    // kernel that uses the tensor cores runs one CTA per SM (the occupancy the runtime reports for a
+    // kernel with tcgen05 instructions), so there a slice is always 32 channels wide: half the CTAs
+    // of 16-channel slices (c2: 120-121 against 125 us per frame), while 64- and 128-channel
+    // slices were slower (129 us; c3 123 against 107 us)
+    t.sw = tc ? SW_WIDE : (t.g.span <= 4 && L.p.c_out <= 32) ? SW_NARROW : SW_WIDE;
     t.nsl = dw ? 1 : (L.p.c_out + t.sw - 1) / t.sw;
     t.zw = dw ? L.p.c_out : t.sw;
     // the tensor-core contraction's weights: [K/8][sw][8] bf16, K padded to the MMA's K step
@@ -1422,10 +1434,9 @@ const void* staged_kernel_of(const Layer& L, int sw)
 }
 
 template <bool WP>
-const void* staged_tc_kernel_of(int sw)
+const void* staged_tc_kernel_of(int)
 {
-    return sw == SW_NARROW ? (const void*)step_local_staged_kernel<__nv_bfloat16, false, SW_NARROW, WP, true>
-                           : (const void*)step_local_staged_kernel<__nv_bfloat16, false, SW_WIDE, WP, true>;
+    return (const void*)step_local_staged_kernel<__nv_bfloat16, false, SW_WIDE, WP, true>;
 }
 
 const void* staged_kernel_of(const Layer& L, int sw, bool wp = false)
@@ -1837,11 +1848,12 @@ cudaError_t launch_step_local(Layer& L, const void* x_t, const void* shortcut, i
         return launch_staged(L, tw, x_t, shortcut, force, nullptr, nullptr, &L.tmap_tx, true);
     if (L.local_staged && !flow) {
         if (!staged_ok(L, &t)) return cudaErrorInvalidValue;
-        // Linked inputs pay only where the grid is more than one wave of resident CTAs: skipped tiles
-        // then take whole waves off the step.  Within one wave every tile runs at once, the step lasts
-        // as long as its slowest (open) tile, and the flag read would only delay each tile's footprint
-        // load by a memory round trip; such a step reads the whole frame instead.
-        if ((long long)L.ntiles * t.nsl <= (long long)L.local_resident) px = psc = nullptr;
+        // Linked inputs pay only where the grid is several waves of resident CTAs: skipped tiles then
+        // take whole waves off the step.  Within one or two waves the step lasts about as long as its
+        // slowest (open) tiles, and the flag read would only delay each tile's footprint load by a
+        // memory round trip (measured: c2 linked 137.7 against 125.2 us unlinked at 1.26 waves); such
+        // a step reads the whole frame instead.
+        if ((long long)L.ntiles * t.nsl <= 2LL * L.local_resident) px = psc = nullptr;
         return launch_staged(L, t, x_t, shortcut, force, px, psc, &L.tmap_fp[cur], false);
     }
     const LocalShape s = choose_shape(L);
