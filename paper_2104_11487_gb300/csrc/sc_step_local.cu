@@ -1605,6 +1605,30 @@ cudaLaunchConfig_t pdl_config(const Layer& L, long long grid, int threads, size_
 
 // The staged form's launch: tm_prev maps the previous input's footprints (x_{t-1}; for a warped
 // step T(x_{t-1}) in fp32, wp = true).
+// CTAs of a staged-form launch resident on the GPU at once, from the SM's register file, shared
+// memory and thread slots (the static limits).  The runtime's occupancy query answers one CTA per SM
+// for the instantiations that contain tcgen05 instructions whatever their size, while the SMs run
+// two or three of them (the limits ncu reports, and the start times of their CTAs).
+cudaError_t staged_resident(const Layer& L, const void* kernel, size_t smem, int* resident)
+{
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, kernel);
+    int regs_sm = 0, smem_sm = 0, smem_reserved = 0, threads_sm = 0;
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, L.device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, L.device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&smem_reserved, cudaDevAttrReservedSharedMemoryPerBlock, L.device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, L.device);
+    if (e != cudaSuccess) return e;
+    // registers are allocated per warp in units of 256
+    const int warp_regs = (fa.numRegs * 32 + 255) / 256 * 256;
+    const int by_regs = regs_sm / (warp_regs * (FT / 32));
+    const int by_smem = smem_sm / (int)(smem + fa.sharedSizeBytes + smem_reserved);
+    const int by_threads = threads_sm / FT;
+    const int per_sm = std::max(1, std::min(by_regs, std::min(by_smem, by_threads)));
+    *resident = L.num_sms * per_sm;
+    return cudaSuccess;
+}
+
 cudaError_t launch_staged(Layer& L, const StagedShape& t, const void* x_t, const void* shortcut, int force,
                           const Layer* px, const Layer* psc, const CUtensorMap* tm_prev, bool wp)
 {
@@ -1751,11 +1775,7 @@ cudaError_t step_local_prepare(Layer& L)
         e = cudaMemsetAsync(L.tile_chg, 0, 2 * (size_t)L.ntiles, L.stream);
         if (e == cudaSuccess) e = alloc_ychg(L);
         if (e == cudaSuccess) e = ensure_dynamic_smem(staged_kernel_of(L, t.sw), t.smem);
-        if (e == cudaSuccess) {
-            int per_sm = 0;
-            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, staged_kernel_of(L, t.sw), FT, t.smem);
-            L.local_resident = L.num_sms * per_sm;
-        }
+        if (e == cudaSuccess) e = staged_resident(L, staged_kernel_of(L, t.sw), t.smem, &L.local_resident);
         // warped steps run the staged form's warped variant, or the general form when it does not fit
         StagedShape tp, tw;
         if (e == cudaSuccess && staged_wp_ok(L, &tp, &tw)) e = ensure_dynamic_smem(staged_kernel_of(L, tw.sw, true), tw.smem);
