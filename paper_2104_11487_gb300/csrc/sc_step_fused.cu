@@ -129,11 +129,12 @@ __device__ __forceinline__ uint4 ld_relaxed_v4(const uint32_t* p)
     return v;
 }
 
-// Between two polls of a warp that waits for published words: back off, and
-// give up (false, the same in every lane) after the time limit or once any
-// CTA raised the abort flag.  `gab` is lane 0's copy of the grid abort flag,
-// loaded together with the polled words (one round trip per poll).
-__device__ __forceinline__ bool poll_backoff(uint64_t t0, int gab, const FusedArgs& a, volatile int* abort, int lane)
+// Between two polls of a warp that waits for published words: give up (false,
+// the same in every lane) after the time limit or once any CTA raised the
+// abort flag.  `gab` is lane 0's copy of the grid abort flag, loaded together
+// with the polled words.  There is no sleep between polls: each poll is
+// already one memory round trip, and a sleep only delays seeing the last word.
+__device__ __forceinline__ bool keep_polling(uint64_t t0, int gab, const FusedArgs& a, volatile int* abort, int lane)
 {
     int give_up = 0;
     if (lane == 0) {
@@ -147,7 +148,6 @@ __device__ __forceinline__ bool poll_backoff(uint64_t t0, int gab, const FusedAr
         if (give_up) *abort = 1;
     }
     give_up = __shfl_sync(0xffffffffu, give_up, 0);
-    if (!give_up) __nanosleep(64);
     return give_up == 0;
 }
 
@@ -361,7 +361,7 @@ __device__ void gate_blocks_role(const FusedArgs& a, FusedShared* sh, volatile i
                         for (int r = 0; r < R; ++r)
                             if ((uint32_t)(v[u][r] >> 32) == a.epoch) need &= ~(1u << (u * R + r));
                     if (!__any_sync(0xffffffffu, need != 0)) break;
-                    if (!(ok = poll_backoff(t0, gab, a, abort, lane))) break;
+                    if (!(ok = keep_polling(t0, gab, a, abort, lane))) break;
                 }
                 if (!ok) return;
 #pragma unroll
@@ -443,7 +443,7 @@ __device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, FS_STAGE
                 for (int b = 0; b < 8; ++b)
                     if ((w[b] >> 1) == a.epoch) need &= ~(1u << b);
                 if (!__any_sync(0xffffffffu, need != 0)) break;
-                if (!(ok = poll_backoff(t0, gab, a, abort, lane))) break;
+                if (!(ok = keep_polling(t0, gab, a, abort, lane))) break;
             }
             if (!ok) break;
             uint32_t bits = 0;
@@ -459,12 +459,17 @@ __device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, FS_STAGE
             }
             const int tot = __shfl_sync(0xffffffffu, incl, 31);
             int e = gprefix + incl - cnt;   // step-wide index of this lane's first open block
+            // the lane's open blocks dealt round-robin: block e of the step goes to CTA e % Q of the slice
+            // (one modulo per lane; the ABI's list is written after the pushes, off the convolution's path)
             uint32_t sel = 0;
-            for (int b = 0; b < 8; ++b) {
-                if (!((bits >> b) & 1u)) continue;
-                if (owner) a.list[e] = n * nb + j0 + b;
-                if (e % Q == q) sel |= 1u << b;
-                ++e;
+            {
+                int r = e % Q;
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    if (!((bits >> b) & 1u)) continue;
+                    if (r == q) sel |= 1u << b;
+                    if (++r == Q) r = 0;
+                }
             }
             if (conv_cta) {
                 // lane 0 pushes the selected blocks in block order, visiting only lanes that hold some
@@ -477,6 +482,11 @@ __device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, FS_STAGE
                     }
                 }
                 ok = __shfl_sync(0xffffffffu, (int)ok, 0) != 0;
+            }
+            if (owner) {
+#pragma unroll
+                for (int b = 0; b < 8; ++b)
+                    if ((bits >> b) & 1u) a.list[e++] = n * nb + j0 + b;
             }
             gprefix += tot;
         }
