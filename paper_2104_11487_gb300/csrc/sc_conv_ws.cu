@@ -42,7 +42,7 @@ constexpr int WS_THREADS = 320;
 constexpr int WS_STAGES = 4;
 
 template <int KS>
-constexpr size_t ws_smem_bytes() { return 1024 + (size_t)ws::Geom<KS, WS_STAGES>::STAGE_BYTES + TC_ZBYTES + 256; }
+constexpr size_t ws_smem_bytes() { return 1024 + (size_t)ws::Geom<KS, WS_STAGES>::STAGE_BYTES + 2 * TC_ZBYTES + 256; }
 
 struct WsArgs {
     const int32_t* list;
@@ -61,7 +61,7 @@ conv_ws_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
     uint8_t* smem = ptx::align_smem_1024(smem_raw);
     uint8_t* sX = smem;
     float* sZ = (float*)(sX + Gm::STAGE_BYTES);
-    ws::Bars* bars = (ws::Bars*)((uint8_t*)sZ + TC_ZBYTES);
+    ws::Bars* bars = (ws::Bars*)((uint8_t*)sZ + 2 * TC_ZBYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     const int slice = blockIdx.x % a.n_slices;
@@ -102,7 +102,7 @@ conv_ws_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant_
     } else if (warp >= 4) {
         ws::residual_role<KS, WS_STAGES>(sX, bars, threadIdx.x - 128, abort, a.err);
     } else {
-        ws::epilogue_role(sZ, bars, tmem, &tm_z, ct, a.nby, a.nbx, threadIdx.x, abort, a.err);
+        ws::epilogue_role(sZ, bars, tmem, &tm_z, ct, a.nby, a.nbx, threadIdx.x, abort, a.err, 2);
     }
 
     ptx::tc_fence_before();

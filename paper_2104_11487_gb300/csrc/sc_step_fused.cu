@@ -85,7 +85,7 @@ struct FusedShared {
 template <int KS>
 constexpr size_t fused_smem_bytes()
 {
-    return 1024 + (size_t)ws::Geom<KS, FS_STAGES>::STAGE_BYTES + (size_t)FS_GATE_WARPS * FS_SLOT + TC_ZBYTES + 256 +
+    return 1024 + (size_t)ws::Geom<KS, FS_STAGES>::STAGE_BYTES + (size_t)FS_GATE_WARPS * FS_SLOT + 2 * TC_ZBYTES + 256 +
            sizeof(FusedShared);
 }
 
@@ -507,7 +507,7 @@ step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_consta
     uint8_t* sX = smem;
     uint8_t* ring = sX + Gm::STAGE_BYTES;
     float* sZ = (float*)(ring + FS_GATE_WARPS * FS_SLOT);
-    ws::Bars* bars = (ws::Bars*)((uint8_t*)sZ + TC_ZBYTES);
+    ws::Bars* bars = (ws::Bars*)((uint8_t*)sZ + 2 * TC_ZBYTES);
     FusedShared* sh = (FusedShared*)((uint8_t*)bars + 256);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -556,7 +556,7 @@ step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_consta
         } else if (warp >= 4) {
             ws::residual_role<KS, FS_STAGES>(sX, bars, threadIdx.x - 128, abort, a.err);
         } else {
-            ws::epilogue_role(sZ, bars, tmem, &tm_z, ct, a.nby, a.nbx, threadIdx.x, abort, a.err);
+            ws::epilogue_role(sZ, bars, tmem, &tm_z, ct, a.nby, a.nbx, threadIdx.x, abort, a.err, 2);
         }
     }
 

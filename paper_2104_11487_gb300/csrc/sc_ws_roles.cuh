@@ -15,9 +15,11 @@
 // the stage, the MMA warp forwards it to the epilogue with its accumulator.
 //
 //   producer (1 thread) : x_empty -> stage_blk, TMA halo rows of x_t, x_{t-1} -> x_full
-//   residual (4 warps)  : x_full -> r = x_t - x_{t-1} in the canonical layout -> r_ready
+//   residual (4 warps)  : x_full -> r = x_t - x_{t-1} in the canonical layout, written over the
+//                         x_{t-1} tile -> r_ready
 //   MMA (1 warp)        : acc_empty, r_ready -> k*k*4 MMAs -> commit x_empty, acc_full; acc_blk -> acc_meta
-//   epilogue (4 warps)  : acc_meta, acc_full -> TMEM -> smem -> TMA reduce-add into z~ -> acc_empty
+//   epilogue (4 warps)  : acc_meta, acc_full -> TMEM -> acc_empty -> smem staging tile (two in turn
+//                         where the kernel has room) -> TMA reduce-add into z~
 //
 // Every wait is bounded (mbar_wait); a role that gives up raises the CTA's
 // abort flag, the others stop at their next wait.
@@ -42,7 +44,8 @@ struct Geom {
     static constexpr int HH = 8 + KS - 1, WW = 8 + KS - 1, TAPS = KS * KS;
     static constexpr int G = (HH * WW) | 1;                  // odd canonical group stride, 16-byte units
     static constexpr int RB = HH * WW * 128;                 // one staged halo tile (one tensor)
-    static constexpr int SB = ((2 * RB + 8 * G * 16 + 1023) / 1024) * 1024;  // stage: x_t, x_{t-1}, r
+    // stage: x_t, then x_{t-1}, over which r is written (r's canonical layout takes 8 * G 16-byte units)
+    static constexpr int SB = ((RB + 8 * G * 16 + 1023) / 1024) * 1024;
     static constexpr int STAGES = NST;
     static constexpr int STAGE_BYTES = NST * SB;
     static constexpr int TAPS_PER_ROUND = STAGE_BYTES / WBYTES;  // weight taps staged per round
@@ -204,7 +207,9 @@ struct Producer {
 };
 
 // Residual warps (tid = 0..127): r = x_t - x_{t-1} (bf16) into the no-swizzle
-// K-major canonical layout [8-channel group][row][col][8 ch], group stride G.
+// K-major canonical layout [8-channel group][row][col][8 ch], group stride G,
+// written over the x_{t-1} tile: every thread forms its residuals in registers,
+// and the four warps meet at named barrier 3 before any of them writes.
 template <int KS, int NST>
 __device__ __forceinline__ void residual_role(uint8_t* sX, Bars* b, int tid, volatile int* abort, int* err)
 {
@@ -218,10 +223,21 @@ __device__ __forceinline__ void residual_role(uint8_t* sX, Bars* b, int tid, vol
         if (id >= 0) {
             const uint4* xt = (const uint4*)(sX + xs * Gm::SB);
             const uint4* xp = (const uint4*)(sX + xs * Gm::SB + Gm::RB);
-            uint4* r = (uint4*)(sX + xs * Gm::SB + 2 * Gm::RB);
+            uint4* r = (uint4*)(sX + xs * Gm::SB + Gm::RB);
             constexpr int NV = Gm::HH * Gm::WW * 8;  // (pixel, 8-channel group) pairs
-#pragma unroll 4
-            for (int v = tid; v < NV; v += 128) r[(v & 7) * Gm::G + (v >> 3)] = bf16x8_sub(xt[v], xp[v]);
+            constexpr int PER = (NV + 127) / 128;
+            uint4 rv[PER];
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int v = tid + 128 * u;
+                if (v < NV) rv[u] = bf16x8_sub(xt[v], xp[v]);
+            }
+            ptx::named_bar_sync(3, 128);
+#pragma unroll
+            for (int u = 0; u < PER; ++u) {
+                const int v = tid + 128 * u;
+                if (v < NV) r[(v & 7) * Gm::G + (v >> 3)] = rv[u];
+            }
             ptx::fence_proxy_async_smem();
         }
         __syncwarp();
@@ -257,7 +273,7 @@ __device__ __forceinline__ void mma_role(uint8_t* sX, Bars* b, uint32_t tmem, vo
         }
         ptx::tc_fence_after();
         const uint32_t d = tmem + ACC_COL + acc * TC_N;
-        const uint64_t b0 = ptx::smem_desc(ptx::smem_u32(sX + xs * Gm::SB + 2 * Gm::RB), Gm::G * 16, Gm::WW * 16, 0);
+        const uint64_t b0 = ptx::smem_desc(ptx::smem_u32(sX + xs * Gm::SB + Gm::RB), Gm::G * 16, Gm::WW * 16, 0);
         if (ptx::elect_one()) {
 #pragma unroll
             for (int t = 0; t < Gm::TAPS; ++t) {
@@ -290,12 +306,15 @@ __device__ __forceinline__ void mma_role(uint8_t* sX, Bars* b, uint32_t tmem, vo
 
 // Epilogue warps 0-3 (tid = 0..127): accumulator (lane = output channel,
 // column = pixel) -> shared memory [pixel][channel] -> TMA reduce-add into
-// z~ at (ct*128, bx*8, by*8, n).
+// z~ at (ct*128, bx*8, by*8, n).  With two staging tiles (zbufs = 2) the tile
+// of block i is refilled once the reduce-add of block i - 2 has read it, so a
+// reduce-add still draining (its z~ lines come from DRAM) does not hold up the
+// next block.
 __device__ __forceinline__ void epilogue_role(float* sZ, Bars* b, uint32_t tmem, const CUtensorMap* tm_z, int ct,
-                                              int nby, int nbx, int tid, volatile int* abort, int* err)
+                                              int nby, int nbx, int tid, volatile int* abort, int* err, int zbufs)
 {
     const int warp = tid >> 5, lane = tid & 31;
-    int acc = 0;
+    int acc = 0, zb = 0;
     uint32_t accph = 0;
     for (;;) {
         if (!group_wait(1, ptx::smem_u32(&b->acc_meta[acc]), accph, abort, err)) break;
@@ -315,22 +334,27 @@ __device__ __forceinline__ void epilogue_role(float* sZ, Bars* b, uint32_t tmem,
         if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&b->acc_empty[acc]));
         if (++acc == 2) { acc = 0; accph ^= 1; }
         const int col = warp * 32 + lane;
-        if (tid == 0) ptx::bulk_wait_group_read0();
+        float* Z = sZ + zb * (TC_N * TC_M);
+        if (tid == 0) {
+            if (zbufs == 2) ptx::bulk_wait_group_read1();
+            else ptx::bulk_wait_group_read0();
+        }
         ptx::named_bar_sync(1, 128);
 #pragma unroll
         for (int p = 0; p < 32; ++p) {
-            sZ[p * TC_M + col] = __uint_as_float(r0[p]);
-            sZ[(p + 32) * TC_M + col] = __uint_as_float(r1[p]);
+            Z[p * TC_M + col] = __uint_as_float(r0[p]);
+            Z[(p + 32) * TC_M + col] = __uint_as_float(r1[p]);
         }
         ptx::fence_proxy_async_smem();
         ptx::named_bar_sync(1, 128);
         if (tid == 0) {
-            ptx::tma_reduce_add_4d(tm_z, ptx::smem_u32(sZ), ct * TC_M, bx * 8, by * 8, n);
+            ptx::tma_reduce_add_4d(tm_z, ptx::smem_u32(Z), ct * TC_M, bx * 8, by * 8, n);
             ptx::bulk_commit_group();
         }
+        if (zbufs == 2) zb ^= 1;
     }
-    // the staging tile must stay valid until the last reduce-add has read it; its writes to z~ complete
-    // with the grid
+    // the staging tiles must stay valid until the last reduce-add has read them; its writes to z~
+    // complete with the grid
     if (tid == 0) ptx::bulk_wait_group_read0();
 }
 
