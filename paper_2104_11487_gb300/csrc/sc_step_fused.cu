@@ -43,12 +43,23 @@
 namespace sc {
 namespace {
 
-constexpr int FS_STAGES = 3;                       // halo stages of the convolution
-constexpr int FS_GATE_WARPS = 8;                   // gate warps = ring slots
+constexpr int FS_MAX_GATE_WARPS = 8;
 constexpr int FS_BG_WARPS = 2;                     // block-gate warps
-constexpr int FS_WARPS = 10 + FS_BG_WARPS + FS_GATE_WARPS;  // 0-3 epilogue, 4-7 residual, 8 producer,
-                                                   // 9 MMA, 10-11 block gate, 12.. gate
-constexpr int FS_THREADS = FS_WARPS * 32;
+
+// Warp roles per CTA: 0-3 epilogue, 4-7 residual, 8 producer, 9 MMA, 10-11
+// block gate, 12.. gate.  NG gate warps (= ring slots), NST halo stages.
+// The sparse step streams with 8 gate warps and 3 halo stages; a forced step
+// (key frame, dense mode: every block open, so the convolution is the work)
+// trades two gate warps' ring slots for a fourth halo stage.
+template <int NG, int NST>
+struct FsCfg {
+    static constexpr int GATE_WARPS = NG, STAGES = NST;
+    static constexpr int WARPS = 10 + FS_BG_WARPS + NG;
+    static constexpr int THREADS = WARPS * 32;
+    static_assert(NG <= FS_MAX_GATE_WARPS, "gate warps");
+};
+using CfgSparse = FsCfg<8, 3>;
+using CfgForced = FsCfg<6, 4>;
 constexpr int FS_SLOT = 8192;                      // ring slot: x_t chunk | x_{t-1} chunk
 constexpr int FS_HALF = FS_SLOT / 2;
 constexpr int FS_FOOT = 16 * 16;                   // block-gate footprint capacity (floats)
@@ -78,14 +89,14 @@ struct FusedArgs {
 };
 
 struct FusedShared {
-    uint64_t g_full[FS_GATE_WARPS];
+    uint64_t g_full[FS_MAX_GATE_WARPS];
     float foot[FS_BG_WARPS][2][FS_FOOT];   // block-gate footprints of pixel norms
 };
 
-template <int KS>
+template <int KS, class C>
 constexpr size_t fused_smem_bytes()
 {
-    return 1024 + (size_t)ws::Geom<KS, FS_STAGES>::STAGE_BYTES + (size_t)FS_GATE_WARPS * FS_SLOT + 2 * TC_ZBYTES + 256 +
+    return 1024 + (size_t)ws::Geom<KS, C::STAGES>::STAGE_BYTES + (size_t)C::GATE_WARPS * FS_SLOT + 2 * TC_ZBYTES + 256 +
            sizeof(FusedShared);
 }
 
@@ -174,7 +185,7 @@ __device__ __forceinline__ float l1_bf16x8(const uint4& a, const uint4& b)
 
 // This CTA's pixels of every stream: [lo, hi) of each stream's h*w, cut into
 // chunks of gch pixels; chunk k (stream n = k / cpn) goes to ring slot and
-// gate warp k % FS_GATE_WARPS.
+// gate warp k % NG.
 struct GateRange {
     int lo, hi, cpn, total;
     __device__ __forceinline__ GateRange(const FusedArgs& a)
@@ -196,7 +207,7 @@ struct GateRange {
 // sum in each lane (row index = the lane's top three sub-lane bits), then
 // plain steps; the pairing is that of a plain xor butterfly, so the sums are
 // bit-identical to it.
-template <int LOG2G>
+template <int LOG2G, int NG>
 __device__ void gate_pixels_role(const FusedArgs& a, FusedShared* sh, const uint8_t* ring, int gw, int lane,
                                  volatile int* abort)
 {
@@ -231,13 +242,13 @@ __device__ void gate_pixels_role(const FusedArgs& a, FusedShared* sh, const uint
     const int my_row = (((sub >> (LOG2G - 1)) & 1) << 2) | (((sub >> (LOG2G - 2)) & 1) << 1) | ((sub >> (LOG2G - 3)) & 1);
     const bool writer = (sub & ((G >> 3) - 1)) == 0;
     uint32_t ph = 0;
-    for (int k = gw; k < R.total; k += FS_GATE_WARPS, ph ^= 1u) {
+    for (int k = gw; k < R.total; k += NG, ph ^= 1u) {
         const int n = k / R.cpn;
         const int p0 = R.lo + (k - n * R.cpn) * CH;
         const int np = min(CH, R.hi - p0);
         const long long base = (long long)n * a.P + p0;
         const uint32_t cm = __ballot_sync(0xffffffffu, chg_next != 0);
-        chg_next = chg_of(k + FS_GATE_WARPS);
+        chg_next = chg_of(k + NG);
         if (!ws::warp_wait(full, ph, abort, a.err)) {
             // the copy in flight may still land: wait for it (bounded) before the CTA can exit
             if (lane == 0) ptx::mbar_wait(full, ph, nullptr, nullptr, ws::WAIT_NS);
@@ -259,9 +270,9 @@ __device__ void gate_pixels_role(const FusedArgs& a, FusedShared* sh, const uint
             d[u] = (av[u].x ^ b.x) | (av[u].y ^ b.y) | (av[u].z ^ b.z) | (av[u].w ^ b.w);
         }
         __syncwarp();
-        if (lane == 0 && k + FS_GATE_WARPS < R.total) {
+        if (lane == 0 && k + NG < R.total) {
             ptx::fence_proxy_async_smem();   // the slot's reads before the copy that overwrites it
-            issue(k + FS_GATE_WARPS);
+            issue(k + NG);
         }
         // transposed butterfly over the pixel's G lanes
         float t4[4], t2[2], t1;
@@ -406,8 +417,8 @@ __device__ void gate_blocks_role(const FusedArgs& a, FusedShared* sh, volatile i
     }
 }
 
-template <int KS>
-__device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, FS_STAGES>& pr, bool conv_cta, int Q, int q,
+template <int KS, int NST>
+__device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, NST>& pr, bool conv_cta, int Q, int q,
                                    volatile int* abort, int lane)
 {
     const int nb = a.nby * a.nbx;
@@ -495,18 +506,19 @@ __device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, FS_STAGE
     if (lane == 0) pr.finish();
 }
 
-template <int KS>
-__global__ void __launch_bounds__(FS_THREADS, 1)
+template <int KS, class C>
+__global__ void __launch_bounds__(C::THREADS, 1)
 step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_constant__ CUtensorMap tm_xp,
                   const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_z,
                   const FusedArgs a)
 {
-    using Gm = ws::Geom<KS, FS_STAGES>;
+    using Gm = ws::Geom<KS, C::STAGES>;
+    constexpr int NG = C::GATE_WARPS, NST = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = ptx::align_smem_1024(smem_raw);
     uint8_t* sX = smem;
     uint8_t* ring = sX + Gm::STAGE_BYTES;
-    float* sZ = (float*)(ring + FS_GATE_WARPS * FS_SLOT);
+    float* sZ = (float*)(ring + NG * FS_SLOT);
     ws::Bars* bars = (ws::Bars*)((uint8_t*)sZ + 2 * TC_ZBYTES);
     FusedShared* sh = (FusedShared*)((uint8_t*)bars + 256);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -518,7 +530,7 @@ step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_consta
 
     if (threadIdx.x == 0) {
         ws::init_barriers(bars);
-        for (int s = 0; s < FS_GATE_WARPS; ++s) ptx::mbar_init(ptx::smem_u32(&sh->g_full[s]), 1);
+        for (int s = 0; s < NG; ++s) ptx::mbar_init(ptx::smem_u32(&sh->g_full[s]), 1);
         ptx::fence_mbar_init();
     }
     if (warp == 9) {
@@ -533,28 +545,28 @@ step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_consta
 
     if (warp >= 10 + FS_BG_WARPS) {
         const int gw = warp - 10 - FS_BG_WARPS;
-        if (a.log2g == 5) gate_pixels_role<5>(a, sh, ring, gw, lane, abort);
-        else if (a.log2g == 4) gate_pixels_role<4>(a, sh, ring, gw, lane, abort);
-        else gate_pixels_role<3>(a, sh, ring, gw, lane, abort);
+        if (a.log2g == 5) gate_pixels_role<5, NG>(a, sh, ring, gw, lane, abort);
+        else if (a.log2g == 4) gate_pixels_role<4, NG>(a, sh, ring, gw, lane, abort);
+        else gate_pixels_role<3, NG>(a, sh, ring, gw, lane, abort);
     } else if (warp >= 10) {
         gate_blocks_role<KS>(a, sh, abort, warp - 10, lane);
     } else {
         // convolution roles: the weight slice goes through the stage area into
         // TMEM first (named barrier 2 over the 10 convolution warps)
         if (conv_cta && warp < 4)
-            ws::load_weight_slice<KS, FS_STAGES>(&tm_w, sX, bars, tmem, a.ci_pad, chunk, ct, threadIdx.x, abort,
+            ws::load_weight_slice<KS, NST>(&tm_w, sX, bars, tmem, a.ci_pad, chunk, ct, threadIdx.x, abort,
                                                  a.err);
         ptx::tc_fence_before();
         ptx::named_bar_sync(2, 320);
         ptx::tc_fence_after();
         if (warp == 8) {
-            ws::Producer<KS, FS_STAGES> pr;
+            ws::Producer<KS, NST> pr;
             if (lane == 0) pr.init(sX, bars, &tm_xt, &tm_xp, abort, a.err, chunk, a.pad, a.nby, a.nbx);
-            conv_producer_role<KS>(a, pr, conv_cta, Q, q, abort, lane);
+            conv_producer_role<KS, NST>(a, pr, conv_cta, Q, q, abort, lane);
         } else if (warp == 9) {
-            ws::mma_role<KS, FS_STAGES>(sX, bars, tmem, abort, a.err);
+            ws::mma_role<KS, NST>(sX, bars, tmem, abort, a.err);
         } else if (warp >= 4) {
-            ws::residual_role<KS, FS_STAGES>(sX, bars, threadIdx.x - 128, abort, a.err);
+            ws::residual_role<KS, NST>(sX, bars, threadIdx.x - 128, abort, a.err);
         } else {
             ws::epilogue_role(sZ, bars, tmem, &tm_z, ct, a.nby, a.nbx, threadIdx.x, abort, a.err, 2);
         }
@@ -569,34 +581,49 @@ step_fused_kernel(const __grid_constant__ CUtensorMap tm_xt, const __grid_consta
     }
 }
 
-template <int KS>
+template <int KS, class C>
 cudaError_t launch_fused_ks(const Layer& L, const CUtensorMap& tm_xt, int prev_index, const FusedArgs& a)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(L.num_sms);
-    cfg.blockDim = dim3(FS_THREADS);
-    cfg.dynamicSmemBytes = fused_smem_bytes<KS>();
+    cfg.blockDim = dim3(C::THREADS);
+    cfg.dynamicSmemBytes = fused_smem_bytes<KS, C>();
     cfg.stream = L.stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, step_fused_kernel<KS>, tm_xt, L.tmap_xrow[prev_index], L.tmap_w, L.tmap_z, a);
+    return cudaLaunchKernelEx(&cfg, step_fused_kernel<KS, C>, tm_xt, L.tmap_xrow[prev_index], L.tmap_w, L.tmap_z,
+                              a);
+}
+
+template <int KS, class C>
+cudaError_t prepare_cfg(const Layer& L)
+{
+    static_assert(fused_smem_bytes<KS, C>() <= 227 * 1024, "shared memory");
+    cudaError_t e = cudaFuncSetAttribute(step_fused_kernel<KS, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)fused_smem_bytes<KS, C>());
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, step_fused_kernel<KS, C>, C::THREADS,
+                                                      fused_smem_bytes<KS, C>());
+    if (e != cudaSuccess) return e;
+    return per_sm >= 1 ? cudaSuccess : cudaErrorCooperativeLaunchTooLarge;
 }
 
 template <int KS>
 cudaError_t prepare_ks(const Layer& L)
 {
-    static_assert(fused_smem_bytes<KS>() <= 227 * 1024, "shared memory");
-    cudaError_t e = cudaFuncSetAttribute(step_fused_kernel<KS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)fused_smem_bytes<KS>());
-    if (e != cudaSuccess) return e;
-    int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, step_fused_kernel<KS>, FS_THREADS,
-                                                      fused_smem_bytes<KS>());
-    if (e != cudaSuccess) return e;
-    return per_sm >= 1 ? cudaSuccess : cudaErrorCooperativeLaunchTooLarge;
+    const cudaError_t e = prepare_cfg<KS, CfgSparse>(L);
+    return e != cudaSuccess ? e : prepare_cfg<KS, CfgForced>(L);
+}
+
+template <int KS>
+cudaError_t launch_ks(const Layer& L, const CUtensorMap& tm_xt, int prev_index, const FusedArgs& a)
+{
+    return a.force ? launch_fused_ks<KS, CfgForced>(L, tm_xt, prev_index, a)
+                   : launch_fused_ks<KS, CfgSparse>(L, tm_xt, prev_index, a);
 }
 
 }  // namespace
@@ -673,7 +700,7 @@ cudaError_t launch_step_fused(Layer& L, const void* x_t, int force)
     a.ci_pad = L.ci_pad;
     a.n_chunks = L.ci_pad / TC_CK;
     a.n_slices = (L.co_pad / TC_M) * a.n_chunks;
-    return L.p.k_h == 3 ? launch_fused_ks<3>(L, tm_xt, cur, a) : launch_fused_ks<1>(L, tm_xt, cur, a);
+    return L.p.k_h == 3 ? launch_ks<3>(L, tm_xt, cur, a) : launch_ks<1>(L, tm_xt, cur, a);
 }
 
 }  // namespace sc

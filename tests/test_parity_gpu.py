@@ -145,6 +145,22 @@ def test_ragged_tail_and_several_tiles(path):
     assert cmp.frames == 6
 
 
+@pytest.mark.parametrize("path", [AUTO, SEPARATE])
+def test_ragged_c256_every_slice(path):
+    """Ragged frame (36x44: the last block row and column are partial) with the
+    headline's 256 input channels (4 input-channel slices summed into z~) and
+    200 output channels (the second 128-channel output slice is partly past
+    c_out, so its boxes are clipped), 6 frames, full z~ every frame."""
+    frames = synth.round_to_bf16(synth.moving_squares_video(91, 6, 36, 44, 256, n_squares=3, size=10))
+    rng = np.random.default_rng(92)
+    w = synth.he_weights(rng, 200, 256, 3, bf16=True)
+    b = synth.round_to_bf16(rng.standard_normal(200).astype(np.float32) * 0.1)
+    spec = LayerSpec(n=1, c_in=256, c_out=200, h=36, w=44, k=3, block=8, eps=0.05)
+    cmp, used = run_single_layer(spec, w, b, [f[None] for f in frames], "bf16", conv_path=path,
+                                 name="ragged c256", expect_fused=FUSED[path])
+    assert used == TENSOR_CORE and cmp.frames == 6
+
+
 @pytest.mark.parametrize("path", [AUTO, SEPARATE, CUDA_CORE, CC_SEPARATE])
 def test_dense_mode_is_dense_conv(path):
     wl = synth.make_workload("c1", T=4)
