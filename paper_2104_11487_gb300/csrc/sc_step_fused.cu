@@ -48,9 +48,13 @@ constexpr int FS_BG_WARPS = 2;                     // block-gate warps
 
 // Warp roles per CTA: 0-3 epilogue, 4-7 residual, 8 producer, 9 MMA, 10-11
 // block gate, 12.. gate.  NG gate warps (= ring slots), NST halo stages.
-// The sparse step streams with 8 gate warps and 3 halo stages; a forced step
-// (key frame, dense mode: every block open, so the convolution is the work)
-// trades two gate warps' ring slots for a fourth halo stage.
+// The sparse step streams with 8 gate warps and 3 halo stages.  In a forced
+// step (key frame, dense mode) every decision is published at once, so the
+// convolution starts at the kernel's start and is the work; the gate only
+// commits x_t beside it, which 2 gate warps finish well before the
+// convolution does, and the six ring slots this frees buy two more halo
+// stages (measured on a dense c4 step: 8 gate warps / 3 stages 129.0 us,
+// 6 / 4 123.5, 3 / 5 120.3, 2 / 5 118.1, 4 / 4 124.1).
 template <int NG, int NST>
 struct FsCfg {
     static constexpr int GATE_WARPS = NG, STAGES = NST;
@@ -59,7 +63,7 @@ struct FsCfg {
     static_assert(NG <= FS_MAX_GATE_WARPS, "gate warps");
 };
 using CfgSparse = FsCfg<8, 3>;
-using CfgForced = FsCfg<6, 4>;
+using CfgForced = FsCfg<2, 5>;
 constexpr int FS_SLOT = 8192;                      // ring slot: x_t chunk | x_{t-1} chunk
 constexpr int FS_HALF = FS_SLOT / 2;
 constexpr int FS_FOOT = 16 * 16;                   // block-gate footprint capacity (floats)

@@ -32,7 +32,7 @@
 namespace sc {
 namespace ws {
 
-constexpr int MAX_STAGES = 4;
+constexpr int MAX_STAGES = 5;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t ACC_COL = 384;   // accumulators at columns 384 and 448
 constexpr uint64_t WAIT_NS = 1000000000ull;
