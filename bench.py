@@ -853,6 +853,17 @@ def main():
         from paper_2104_11487_gb300 import skipconv_step_host, skipconv_step_host_async, skipconv_sync
         host = [f.cpu().pin_memory() for f in frames]
         zh = [torch.empty((N_STREAMS, H, W, C), dtype=torch.float32).pin_memory() for _ in range(2)]
+        # one untimed round trip through every pinned buffer first: the first copies out of freshly pinned
+        # host memory were measured at 3-5 ms per 192 MiB step against 1.07 ms once the buffers had been
+        # used, and a caller allocates its pinned buffers once
+        scratch = torch.empty_like(frames[0])
+        for hb in host:
+            scratch.copy_(hb, non_blocking=True)
+        zscratch = torch.empty((N_STREAMS, H, W, C), dtype=torch.float32, device="cuda")
+        for zb in zh:
+            zb.copy_(zscratch, non_blocking=True)
+        torch.cuda.synchronize()
+        del scratch, zscratch
         # synchronous calls: each step uploads, steps, downloads and waits
         layer.reset()
         for i in range(args.warmup + 1):

@@ -322,10 +322,13 @@ int skipconv_create(const skipconv_params* params, const void* weights_oihw, con
         e = A.dev((void**)&L.w_tc, (size_t)L.co_pad * L.p.k_h * L.p.k_w * L.ci_pad * sizeof(__nv_bfloat16));
     if (e == cudaSuccess) e = A.dev((void**)&w_l1_dev, sizeof(double));
     if (e == cudaSuccess) {
-        e = cudaHostAlloc((void**)&L.err_host, sizeof(int), cudaHostAllocMapped);
+        // the device error word and, a cache line further, the fused step's open-block hint
+        e = cudaHostAlloc((void**)&L.err_host, 32 * sizeof(int), cudaHostAllocMapped);
         if (e == cudaSuccess) {
-            *L.err_host = 0;
+            memset(L.err_host, 0, 32 * sizeof(int));
             e = cudaHostGetDevicePointer((void**)&L.err_dev, L.err_host, 0);
+            L.open_hint_host = L.err_host + 16;
+            L.open_hint_dev = L.err_dev + 16;
         }
     }
     L.state_bytes = A.bytes;

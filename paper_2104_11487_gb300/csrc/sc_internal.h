@@ -55,6 +55,8 @@ struct Layer {
     // error word: pinned, mapped host memory
     int* err_host;
     int* err_dev;
+    int* open_hint_host;    // fused step: the last sparse step's open-block count, written by the kernel into
+    int* open_hint_dev;     // mapped host memory (same allocation as err_host); picks the next launch's form
 
     // profiling (host): launch counts per kernel kind, optional event pairs
     long long launches[SKIPCONV_PROFILE_KINDS];

@@ -48,13 +48,16 @@ constexpr int FS_BG_WARPS = 2;                     // block-gate warps
 
 // Warp roles per CTA: 0-3 epilogue, 4-7 residual, 8 producer, 9 MMA, 10-11
 // block gate, 12.. gate.  NG gate warps (= ring slots), NST halo stages.
-// The sparse step streams with 8 gate warps and 3 halo stages.  In a forced
-// step (key frame, dense mode) every decision is published at once, so the
-// convolution starts at the kernel's start and is the work; the gate only
-// commits x_t beside it, which 2 gate warps finish well before the
-// convolution does, and the six ring slots this frees buy two more halo
-// stages (measured on a dense c4 step: 8 gate warps / 3 stages 129.0 us,
-// 6 / 4 123.5, 3 / 5 120.3, 2 / 5 118.1, 4 / 4 124.1).
+// A sparse step streams with 8 gate warps and 3 halo stages.  When the last
+// sparse step opened at least 3/8 of the blocks, the convolution is most of
+// the work and 6 gate warps / 4 halo stages pay instead (c4, us per step at
+// 10 / 25 / 50 / 100 % density: 8 / 3 43.2, 55.2, 82.1, 132.7; 6 / 4 49.5,
+// 57.8, 79.9, 125.7).  In a forced step (key frame, dense mode) every
+// decision is published at once, so the convolution starts at the kernel's
+// start; the gate only commits x_t beside it, which 2 gate warps finish well
+// before the convolution does, and the six ring slots this frees buy two more
+// halo stages (a dense c4 step: 8 / 3 129.0 us, 6 / 4 123.5, 3 / 5 120.3,
+// 2 / 5 118.1, 4 / 4 124.1).
 template <int NG, int NST>
 struct FsCfg {
     static constexpr int GATE_WARPS = NG, STAGES = NST;
@@ -63,6 +66,7 @@ struct FsCfg {
     static_assert(NG <= FS_MAX_GATE_WARPS, "gate warps");
 };
 using CfgSparse = FsCfg<8, 3>;
+using CfgBusy = FsCfg<6, 4>;
 using CfgForced = FsCfg<2, 5>;
 constexpr int FS_SLOT = 8192;                      // ring slot: x_t chunk | x_{t-1} chunk
 constexpr int FS_HALF = FS_SLOT / 2;
@@ -82,6 +86,7 @@ struct FusedArgs {
     uint32_t* gtag;        // per gate block: (epoch << 1) | open
     int32_t* list;
     int32_t* count;        // this step's open-block count (the ABI's view)
+    int* hint;             // mapped host word: this step's open-block count (sparse steps), a launch hint
     int* gabort;           // grid-wide abort flag
     uint32_t epoch;        // this step's tag, 1 .. 2^31 - 1
     float thr;
@@ -505,7 +510,10 @@ __device__ void conv_producer_role(const FusedArgs& a, ws::Producer<KS, NST>& pr
             }
             gprefix += tot;
         }
-        if (n == a.n - 1 && lane == 0 && ok && (int)blockIdx.x == n % (int)gridDim.x) *a.count = gprefix;
+        if (n == a.n - 1 && lane == 0 && ok && (int)blockIdx.x == n % (int)gridDim.x) {
+            *a.count = gprefix;
+            if (!a.force) *(volatile int*)a.hint = gprefix;
+        }
     }
     if (lane == 0) pr.finish();
 }
@@ -619,15 +627,22 @@ cudaError_t prepare_cfg(const Layer& L)
 template <int KS>
 cudaError_t prepare_ks(const Layer& L)
 {
-    const cudaError_t e = prepare_cfg<KS, CfgSparse>(L);
+    cudaError_t e = prepare_cfg<KS, CfgSparse>(L);
+    if (e == cudaSuccess) e = prepare_cfg<KS, CfgBusy>(L);
     return e != cudaSuccess ? e : prepare_cfg<KS, CfgForced>(L);
 }
 
+// The launch's form: forced steps one, sparse steps another after a sparse step that opened at least
+// 3/8 of the blocks.  The hint is the count the last finished sparse step wrote into mapped host memory
+// (a launch queued behind a running step reads the one before: it only chooses the form).
 template <int KS>
 cudaError_t launch_ks(const Layer& L, const CUtensorMap& tm_xt, int prev_index, const FusedArgs& a)
 {
-    return a.force ? launch_fused_ks<KS, CfgForced>(L, tm_xt, prev_index, a)
-                   : launch_fused_ks<KS, CfgSparse>(L, tm_xt, prev_index, a);
+    if (a.force) return launch_fused_ks<KS, CfgForced>(L, tm_xt, prev_index, a);
+    const long long nblk = (long long)a.n * a.nby * a.nbx;
+    const int last_open = *(volatile const int*)L.open_hint_host;
+    return 8LL * last_open >= 3LL * nblk ? launch_fused_ks<KS, CfgBusy>(L, tm_xt, prev_index, a)
+                                         : launch_fused_ks<KS, CfgSparse>(L, tm_xt, prev_index, a);
 }
 
 }  // namespace
@@ -689,6 +704,7 @@ cudaError_t launch_step_fused(Layer& L, const void* x_t, int force)
     a.gtag = L.gtag;
     a.list = L.list;
     a.count = step_count(L);
+    a.hint = L.open_hint_dev;
     a.gabort = L.sched;
     a.epoch = L.epoch;
     a.thr = L.gate_thr;
