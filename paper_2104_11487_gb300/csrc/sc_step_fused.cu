@@ -6,7 +6,7 @@
 // blocks (Eq. 3) -- run concurrently in different warps of every CTA and are
 // pipelined over the independent streams n = 0, 1, ...:
 //
-//   8 gate warps
+//   gate warps (8, or fewer in the busier launch forms below)
 //       stream this CTA's share of every stream's pixels, in stream order,
 //       through shared-memory slots that each warp refills by bulk copies (no
 //       registers or L1 held by loads in flight); form r_t = x_t - x_{t-1}
@@ -24,7 +24,11 @@
 //       partial products into z~ (TMA reduce-add).
 //
 // So the convolution of stream n overlaps the streaming of the streams after
-// it and reads its halo rows while they are still in L2.
+// it and reads its halo rows while they are still in L2.  The kernel is
+// instantiated in three forms that split the shared memory differently
+// between the gate's ring slots and the convolution's halo stages (FsCfg
+// below): the sparse form, a form for steps expected to open many blocks,
+// and a form for forced steps.
 //
 // Hand-off between CTAs carries its own readiness: a published norm is one
 // 64-bit word (step epoch, fp32 norm) and a gate decision one 32-bit word
