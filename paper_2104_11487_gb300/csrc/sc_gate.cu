@@ -499,6 +499,39 @@ __global__ void __launch_bounds__(256) gate_pixel_gumbel_vec_kernel(
 // records a timeout in the error word.
 constexpr int GS_WARPS = 8;
 constexpr int GS_ROWS = 8;                       // pixels per chunk
+
+// Packed pairs of fp32 values (one 64-bit register) and the sm_100-family
+// paired arithmetic on them: each lane of a pair is the IEEE fp32 operation
+// with round to nearest, exactly what the scalar instruction computes, in
+// half the instructions.
+__device__ __forceinline__ unsigned long long f2pack(float lo, float hi)
+{
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2unpack(unsigned long long v, float& lo, float& hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long f2sub(unsigned long long a, unsigned long long b)
+{
+    unsigned long long d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long f2mul(unsigned long long a, unsigned long long b)
+{
+    unsigned long long d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long f2fma(unsigned long long a, unsigned long long b, unsigned long long c)
+{
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
 constexpr int GS_HALF = GS_ROWS * 512;           // one frame's chunk
 constexpr int GS_SLOT = 2 * GS_HALF;
 constexpr int GS_NSLOT = 2;                      // chunks in flight per warp
@@ -565,7 +598,9 @@ __global__ void __launch_bounds__(GS_WARPS * 32, 1) gate_pixel_gumbel_stream_ker
         }
         const uint4* sx = reinterpret_cast<const uint4*>(slots + q * GS_SLOT);
         const uint4* sp = reinterpret_cast<const uint4*>(slots + q * GS_SLOT + GS_HALF);
-        float r[GS_ROWS][8];
+        // residuals of rows 2i and 2i+1 packed in pairs: r2[i][j] = (r[2i][j], r[2i+1][j])
+        unsigned long long r2[GS_ROWS / 2][8];
+        float fa_even[8], fb_even[8];
         uint32_t chg_rows = 0;   // bit row: the pixel changed
 #pragma unroll
         for (int row = 0; row < GS_ROWS; ++row) {
@@ -582,8 +617,17 @@ __global__ void __launch_bounds__(GS_WARPS * 32, 1) gate_pixel_gumbel_stream_ker
             float fa[8], fb[8];
             unpack8(av, fa, (const T*)nullptr);
             unpack8(bv, fb, (const T*)nullptr);
+            if ((row & 1) == 0) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) r[row][j] = fa[j] - fb[j];
+                for (int j = 0; j < 8; ++j) {
+                    fa_even[j] = fa[j];
+                    fb_even[j] = fb[j];
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    r2[row / 2][j] = f2sub(f2pack(fa_even[j], fa[j]), f2pack(fb_even[j], fb[j]));
+            }
         }
         __syncwarp();
         if (lane == 0 && k + GS_NSLOT * ks < nch) {
@@ -593,25 +637,29 @@ __global__ void __launch_bounds__(GS_WARPS * 32, 1) gate_pixel_gumbel_stream_ker
         phases ^= 1u << q;
         q = q + 1 == GS_NSLOT ? 0 : q + 1;
         // the chunk's tap products: v[row * 9 + t] = sum over this lane's channels of phi[t][c] r[c]
+        // (the products and sums of each row are the scalar sequence mul, fma, fma, ...: two rows per instruction)
         float v[GS_ROWS * GUMBEL_MAX_TAPS];
 #pragma unroll
         for (int t = 0; t < GUMBEL_MAX_TAPS; ++t) {
             const float4 w0 = *reinterpret_cast<const float4*>(sphi + t * C + lane * VX);
             const float4 w1 = VX == 8 ? *reinterpret_cast<const float4*>(sphi + t * C + lane * VX + 4)
                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            const unsigned long long p0 = f2pack(w0.x, w0.x), p1 = f2pack(w0.y, w0.y), p2 = f2pack(w0.z, w0.z),
+                                     p3 = f2pack(w0.w, w0.w), p4 = f2pack(w1.x, w1.x), p5 = f2pack(w1.y, w1.y),
+                                     p6 = f2pack(w1.z, w1.z), p7 = f2pack(w1.w, w1.w);
 #pragma unroll
-            for (int row = 0; row < GS_ROWS; ++row) {
-                float a = w0.x * r[row][0];
-                a = fmaf(w0.y, r[row][1], a);
-                a = fmaf(w0.z, r[row][2], a);
-                a = fmaf(w0.w, r[row][3], a);
+            for (int i = 0; i < GS_ROWS / 2; ++i) {
+                unsigned long long a = f2mul(p0, r2[i][0]);
+                a = f2fma(p1, r2[i][1], a);
+                a = f2fma(p2, r2[i][2], a);
+                a = f2fma(p3, r2[i][3], a);
                 if (VX == 8) {
-                    a = fmaf(w1.x, r[row][4], a);
-                    a = fmaf(w1.y, r[row][5], a);
-                    a = fmaf(w1.z, r[row][6], a);
-                    a = fmaf(w1.w, r[row][7], a);
+                    a = f2fma(p4, r2[i][4], a);
+                    a = f2fma(p5, r2[i][5], a);
+                    a = f2fma(p6, r2[i][6], a);
+                    a = f2fma(p7, r2[i][7], a);
                 }
-                v[row * GUMBEL_MAX_TAPS + t] = a;
+                f2unpack(a, v[(2 * i) * GUMBEL_MAX_TAPS + t], v[(2 * i + 1) * GUMBEL_MAX_TAPS + t]);
             }
         }
         // transposed butterfly: each halving exchange keeps half of the rows, until one row's 9 sums are
