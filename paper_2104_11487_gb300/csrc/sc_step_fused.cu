@@ -47,7 +47,7 @@
 namespace sc {
 namespace {
 
-constexpr int FS_MAX_GATE_WARPS = 8;
+constexpr int FS_MAX_GATE_WARPS = 8;              // gate warps of the widest form (barrier slots)
 constexpr int FS_BG_WARPS = 2;                     // block-gate warps
 
 // Warp roles per CTA: 0-3 epilogue, 4-7 residual, 8 producer, 9 MMA, 10-11
@@ -109,8 +109,8 @@ struct FusedShared {
 template <int KS, class C>
 constexpr size_t fused_smem_bytes()
 {
-    return 1024 + (size_t)ws::Geom<KS, C::STAGES>::STAGE_BYTES + (size_t)C::GATE_WARPS * FS_SLOT + 2 * TC_ZBYTES + 256 +
-           sizeof(FusedShared);
+    return 1024 + (size_t)ws::Geom<KS, C::STAGES>::STAGE_BYTES + (size_t)C::GATE_WARPS * FS_SLOT + 2 * TC_ZBYTES +
+           256 + sizeof(FusedShared);
 }
 
 __device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p)
