@@ -239,7 +239,7 @@ def run_layer_timed(layer, frames, warmup, steps, flush, torch, profile=False):
 
 CONV_PATH = {"fused": 0, "separate": 3}   # AUTO (one fused launch per step) / TENSOR_CORE_SEPARATE
 LAUNCH_FORMS = {0: "separate gate and convolution launches", 1: "one cooperative tensor-core launch",
-                2: "one CUDA-core launch (a CTA per tile of gate blocks)"}
+                2: "one launch, a CTA per tile of gate blocks (contraction on the path named)"}
 
 
 GATES = {"input": 0, "output": 2, "gumbel": 3}   # Input-Norm (mean), Output-Norm, Gumbel (Eq. 8)

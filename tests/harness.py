@@ -98,7 +98,8 @@ def run_single_layer(spec, w, bias, frames, dtype, dense_mode=False, conv_path=0
     """Drive one layer over `frames` (iterable of float32 [n,h,w,c] arrays) on
     both sides; returns the Compare record and the conv path used.
     expect_fused: None, or the info.fused value the layer must report (0 separate
-    launches, 1 one cooperative tensor-core launch, 2 one CUDA-core launch).
+    launches, 1 one cooperative tensor-core launch, 2 one launch with a CTA per
+    tile of gate blocks).
     reset_at: frames before which both sides are reset; ref_reset_at: frames
     before which only the oracle is reset (the GPU layer resets itself through
     key_interval)."""

@@ -41,7 +41,7 @@ def _frames(case):
 
 
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-def test_noalloc_gate_matches_step_gate(case):
+def test_noalloc_gate_matches_the_oracle_and_the_step_gate(case):
     import torch
     from paper_2104_11487_gb300 import SkipConvLayer, skipconv_gate_noalloc
     name, n, h, w, c, k, stride, pad, block, eps, gate, dtype, video = case
