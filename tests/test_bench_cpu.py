@@ -1,7 +1,8 @@
 """The benchmark's arithmetic, on the CPU: the algorithmic bytes and FLOPs of
 a c4 step (both frames read in full, the commit of changed pixels, the fp32
 z read-modify-write of the open blocks, the weights; 2 FLOPs per MAC of the
-open blocks), the roofline time they give, and the replica aggregation."""
+open blocks), the roofline time they give, the replica aggregation, and the
+lookup of a kernel's DRAM traffic in its ncu summary."""
 import bench
 
 
@@ -46,3 +47,24 @@ def test_reference_arm_prints_the_contract_line():
                            "d2h_bytes_per_step": 0}
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["cpu_baseline"]["value"] == line["value"]
+
+
+def test_traffic_is_read_only_while_the_profiled_sources_are_unchanged(tmp_path, monkeypatch):
+    """The roofline's `traffic` comes from a committed ncu summary, and only while the sha256 it records
+    is that of the kernel's current source files; otherwise (or with no summary) it is None."""
+    import hashlib
+    name, srcs = bench.PROFILE_FILES["step_fused"]
+    csrc = tmp_path / "paper_2104_11487_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for i, f in enumerate(srcs):
+        (csrc / f).write_bytes(b"source %d\n" % i)
+    (tmp_path / "profiles").mkdir()
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.traffic_from_profiles("step_fused") is None        # no summary
+    digest = hashlib.sha256(b"".join(b"source %d\n" % i for i in range(len(srcs)))).hexdigest()
+    summary = tmp_path / "profiles" / ("%s_c4_d10.md" % name)
+    summary.write_text("# x\n\nsource_sha256: %s (files)\ndram_bytes_per_launch: 158153472 (read + write)\n" % digest)
+    assert bench.traffic_from_profiles("step_fused") == 158153472.0
+    (csrc / srcs[0]).write_bytes(b"source 0, edited\n")             # the kernel changed since the capture
+    assert bench.traffic_from_profiles("step_fused") is None
+    assert bench.traffic_from_profiles("no_such_kernel") is None
