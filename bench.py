@@ -136,18 +136,29 @@ class Clocks:
         except Exception:
             self.proc.kill()
         self.f.close()
+        with open(self.path) as f:
+            return self.summarise(f)
+
+    @staticmethod
+    def summarise(lines):
+        """Median and maximum SM clock, maximum power and the throttle reasons seen active, from
+        nvidia-smi's csv,noheader,nounits lines of the query Q (lines it could not measure are skipped)."""
         sm, smax, reasons, power = [], [], set(), []
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for line in open(self.path):
+        for line in lines:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
             try:
-                sm.append(float(parts[1]))
-                smax.append(float(parts[2]))
-                power.append(float(parts[3]))
+                clk, clk_max = float(parts[1]), float(parts[2])
             except ValueError:
                 continue
+            sm.append(clk)
+            smax.append(clk_max)
+            try:
+                power.append(float(parts[3]))
+            except ValueError:
+                pass
             for nm, v in zip(names, parts[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(nm)

@@ -1,8 +1,9 @@
 """The benchmark's arithmetic, on the CPU: the algorithmic bytes and FLOPs of
 a c4 step (both frames read in full, the commit of changed pixels, the fp32
 z read-modify-write of the open blocks, the weights; 2 FLOPs per MAC of the
-open blocks), the roofline time they give, the replica aggregation, and the
-lookup of a kernel's DRAM traffic in its ncu summary."""
+open blocks), the roofline time they give, the replica aggregation, the
+lookup of a kernel's DRAM traffic in its ncu summary, and the summary of the
+clock samples taken during the timed steps."""
 import bench
 
 
@@ -68,3 +69,23 @@ def test_traffic_is_read_only_while_the_profiled_sources_are_unchanged(tmp_path,
     (csrc / srcs[0]).write_bytes(b"source 0, edited\n")             # the kernel changed since the capture
     assert bench.traffic_from_profiles("step_fused") is None
     assert bench.traffic_from_profiles("no_such_kernel") is None
+
+
+def test_clock_samples_summary():
+    """The clocks key of the bench line: the median SM clock under load, the highest maximum clock, and
+    every throttle reason nvidia-smi reported active in any sample (a run that saw a thermal or hardware
+    slowdown is one to reject); samples it could not measure are skipped, a missing power reading only
+    drops the power."""
+    lines = [
+        "0, 2070, 2070, 455.1, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n",
+        "0, 1980, 2070, 601.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n",
+        "0, 2055, 2070, [N/A], 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n",
+        "0, [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]\n",
+        "garbage\n",
+    ]
+    c = bench.Clocks.summarise(lines)
+    assert c["samples"] == 3 and c["sm_mhz"] == 2055.0 and c["sm_max_mhz"] == 2070.0
+    assert c["power_w_max"] == 601.0 and c["reasons"] == ["sw_power_cap"]
+    hot = bench.Clocks.summarise(["0, 1500, 2070, 700, 0x48, Active, Active, Not Active, Not Active\n"])
+    assert hot["reasons"] == ["hw_slowdown", "hw_thermal_slowdown"]
+    assert bench.Clocks.summarise([])["sm_mhz"] is None
